@@ -1,0 +1,178 @@
+/*
+ * vcs.h - C ABI of libvcs.so, the GB300 (sm_103a) hot path of Visual Context
+ * Segmentation (arXiv 2607.11185, Sec. 3.4, Algorithm 1, App. C.1).
+ *
+ * A GUI trajectory of T steps (screenshot tokens followed by response tokens
+ * per step) is cut into training segments that keep a sliding window of the
+ * most recent screenshots as image tokens and carry the earlier steps as text
+ * (Algorithm 1).  The library builds the packed segment layout, gathers the
+ * bf16 Q/K/V rows of every segment token from trajectory-layout tensors, and
+ * runs causal (per-segment) grouped-query softmax attention forward and
+ * backward over the packed segments.
+ *
+ * Conventions shared by every call:
+ *   - Plain C, no allocation, no global state: every buffer is owned by the
+ *     caller.  Device pointers must point to memory of the current CUDA
+ *     device.  Tensors are contiguous, row-major, 16-byte aligned.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default).
+ *     Every call is asynchronous on that stream.
+ *   - The return value is a vcs_status.  Argument errors that the host can
+ *     see are returned before anything is launched.  Errors that only the
+ *     device can see (inconsistent offsets, out-of-range indices, too-small
+ *     capacities, a bounded wait that gave up) are written as a non-zero
+ *     vcs_status into a device-visible int32 status word named by each call;
+ *     the offending work is skipped, never trapped.  The caller reads that
+ *     word after synchronising.
+ *   - Counts of tokens, steps and segments are limited to INT32_MAX.
+ *
+ * Step model (the readings of the paper that the layout follows):
+ *   step t of a trajectory contributes step_img[t] screenshot tokens followed
+ *   by step_txt[t] response tokens; the trajectory token buffer is the
+ *   concatenation of the steps, trajectories are concatenated in order.  A
+ *   segment holds at most keep + window screenshots (Algorithm 1's prune
+ *   trigger n_img > K + delta, with K = keep and delta = window).  The first
+ *   segment takes steps 1..min(keep+window, T); each later one takes the next
+ *   `window` steps as new steps and retains the `keep` steps before them with
+ *   their screenshots.  Earlier steps appear as their response tokens only.
+ *   Only the response tokens of a segment's new steps are trainable (each
+ *   response is optimised exactly once, App. C.1).  keep = 0 gives a window
+ *   of the `window` most recent screenshots; keep = 0, window = 1 gives
+ *   step-wise decomposition (Sec. 1); keep + window >= T gives one segment
+ *   per trajectory.
+ */
+#ifndef VCS_H_
+#define VCS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum vcs_status {
+  VCS_OK = 0,
+  VCS_ERR_INVALID_ARG = 1,     /* null pointer, negative count, misaligned pointer, bad window */
+  VCS_ERR_UNSUPPORTED = 2,     /* head_dim not 64/128, hq not a multiple of hkv, ... */
+  VCS_ERR_CAPACITY = 3,        /* an output buffer is smaller than the layout needs */
+  VCS_ERR_OVERFLOW = 4,        /* a token count does not fit int32 */
+  VCS_ERR_CUDA = 5,            /* a CUDA runtime or driver call failed */
+  VCS_ERR_DEVICE_CHECK = 6,    /* a kernel found inconsistent input data */
+  VCS_ERR_DEVICE_TIMEOUT = 7,  /* a bounded device-side wait gave up */
+  VCS_ERR_WORKSPACE = 8        /* workspace pointer NULL or smaller than the size query */
+} vcs_status;
+
+/* Sizes of a segment layout, written by the device.  Must live in device
+ * memory or in pinned (mapped) host memory. */
+typedef struct vcs_sizes {
+  int64_t num_segments;
+  int64_t num_tokens;
+  int32_t max_seqlen;
+  int32_t status;              /* vcs_status of device-side checks, 0 = OK */
+} vcs_sizes;
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char* vcs_status_string(int32_t status);
+
+/* Library version / build string (static storage). */
+const char* vcs_version(void);
+
+/* ------------------------------------------------------------------------ *
+ * Segment builder (Sec. 3.4, Algorithm 1; App. C.1)
+ * ------------------------------------------------------------------------ */
+
+/* Workspace bytes for vcs_plan_segments / vcs_build_segments. */
+size_t vcs_segments_workspace_size(int32_t num_traj, int64_t num_steps);
+
+/* Phase 1: sizes of the segment layout.
+ *   cu_steps  [num_traj+1] int32 device: step range of each trajectory
+ *             (cu_steps[0] = 0, non-decreasing, cu_steps[num_traj] = num_steps)
+ *   step_img  [num_steps] int32 device: screenshot tokens of each step (>= 0)
+ *   step_txt  [num_steps] int32 device: response tokens of each step (>= 0)
+ *   window    delta of Algorithm 1 (>= 1): new screenshots per segment
+ *   keep      K of Algorithm 1 (>= 0): screenshots retained across a prune
+ *   sizes     device-visible output: segment count, segment-token count,
+ *             longest segment, device status (VCS_ERR_DEVICE_CHECK for
+ *             inconsistent cu_steps or negative counts, VCS_ERR_OVERFLOW when
+ *             a token count exceeds INT32_MAX)
+ *   ws        device workspace of vcs_segments_workspace_size() bytes
+ * Asynchronous: synchronise `stream` before reading *sizes. */
+vcs_status vcs_plan_segments(const int32_t* cu_steps, int32_t num_traj, int64_t num_steps,
+                             const int32_t* step_img, const int32_t* step_txt,
+                             int32_t window, int32_t keep, vcs_sizes* sizes,
+                             void* ws, size_t ws_bytes, void* stream);
+
+/* Phase 2: the token-level layout (same inputs as phase 1).
+ *   cu_seqlens    [num_segments+1] int32: segment boundaries in the packed buffer
+ *   seg_traj      [num_segments] int32 or NULL: trajectory of each segment
+ *   tok_gather    [num_tokens] int32: index into the trajectory token buffer
+ *   tok_src_step  [num_tokens] int32: global step index (into step_img/step_txt)
+ *   tok_pos       [num_tokens] int32: position in the segment, 0..L-1
+ *   tok_loss_mask [num_tokens] uint8 or NULL: 1 on trainable response tokens
+ *   seg_capacity / tok_capacity: element capacities of the segment / token
+ *   arrays.  If the layout needs more, nothing is written past the capacity
+ *   and sizes->status becomes VCS_ERR_CAPACITY.  sizes receives the same
+ *   values as in phase 1. */
+vcs_status vcs_build_segments(const int32_t* cu_steps, int32_t num_traj, int64_t num_steps,
+                              const int32_t* step_img, const int32_t* step_txt,
+                              int32_t window, int32_t keep,
+                              int64_t seg_capacity, int64_t tok_capacity,
+                              int32_t* cu_seqlens, int32_t* seg_traj, int32_t* tok_gather,
+                              int32_t* tok_src_step, int32_t* tok_pos, uint8_t* tok_loss_mask,
+                              vcs_sizes* sizes, void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ *
+ * Gather: packed segment rows from trajectory rows (the re-tokenised fresh
+ * stream of Algorithm 1 re-uses trajectory tokens).
+ *   q_traj [traj_tokens, hq, d], k_traj / v_traj [traj_tokens, hkv, d] bf16 device
+ *   tok_gather [num_tokens] int32 device (from vcs_build_segments)
+ *   q [num_tokens, hq, d], k / v [num_tokens, hkv, d] bf16 device outputs
+ *   dev_status  int32 device word or NULL: set to VCS_ERR_DEVICE_CHECK if a
+ *               gather index is outside [0, traj_tokens) (that row is skipped)
+ * k_traj/v_traj/k/v may all be NULL to gather Q only.  Bit-exact copy.
+ * ------------------------------------------------------------------------ */
+vcs_status vcs_gather(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
+                      const int32_t* tok_gather, int64_t num_tokens, int32_t hq, int32_t hkv, int32_t d,
+                      void* q, void* k, void* v, int32_t* dev_status, void* stream);
+
+/* ------------------------------------------------------------------------ *
+ * Attention over packed segments.  Token i of segment s attends to the
+ * tokens j of the same segment with j <= i (causal), query head h uses
+ * key/value head h / (hq / hkv).  softmax_scale <= 0 selects 1/sqrt(d).
+ * Layouts: q, o, dout, dq [num_tokens, hq, d]; k, v, dk, dv
+ * [num_tokens, hkv, d]; all bf16.  lse [hq, num_tokens] fp32, natural log.
+ * cu_seqlens [num_segments+1] int32 device, non-decreasing from 0 to
+ * num_tokens, every segment at most max_seqlen long.  Supported: d in
+ * {64, 128}, hq % hkv == 0, num_tokens < 2^31.  The workspace starts with a
+ * 256-byte header whose first int32 is the device status word
+ * (VCS_ERR_DEVICE_CHECK for inconsistent cu_seqlens, VCS_ERR_DEVICE_TIMEOUT
+ * for a wait that gave up); every call clears it first.
+ * ------------------------------------------------------------------------ */
+
+size_t vcs_attn_fwd_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                                   int32_t hq, int32_t hkv, int32_t d);
+
+/* Forward: o = softmax(scale q k^T, causal within the segment) v, and lse. */
+vcs_status vcs_attn_fwd(const void* q, const void* k, const void* v, const int32_t* cu_seqlens,
+                        int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                        int32_t hq, int32_t hkv, int32_t d, float softmax_scale,
+                        void* o, float* lse, void* ws, size_t ws_bytes, void* stream);
+
+size_t vcs_attn_bwd_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                                   int32_t hq, int32_t hkv, int32_t d);
+
+/* Backward: dq, dk, dv of sum(o * dout), given q, k, v, the forward's o and lse.
+ * dk / dv sum over the hq / hkv query heads that share a key/value head.
+ * The workspace also holds an fp32 dq accumulator and the row terms
+ * D = rowsum(dout * o). */
+vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                        const void* dout, const int32_t* cu_seqlens, int32_t num_segments,
+                        int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
+                        float softmax_scale, void* dq, void* dk, void* dv,
+                        void* ws, size_t ws_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VCS_H_ */

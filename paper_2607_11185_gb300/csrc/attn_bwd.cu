@@ -1,0 +1,476 @@
+// attn_bwd.cu - backward of the packed-segment causal GQA attention, sm_103a.
+//
+// For an upstream gradient dO of o_i = sum_j P_ij v_j (P the causal softmax of
+// s_ij = scale <q_i, k_j> within one segment):
+//   D_i   = <dO_i, o_i>
+//   dP_ij = <dO_i, v_j>,   dS_ij = P_ij (dP_ij - D_i)
+//   dq_i  = scale sum_j dS_ij k_j
+//   dk_j  = scale sum_{h in group} sum_i dS_ij q_i
+//   dv_j  = sum_{h in group} sum_i P_ij dO_i
+// P is recomputed from the forward's log-sum-exp: P_ij = exp(s_ij - lse_i).
+//
+// Three kernels on the caller's stream:
+//   bwd_pre     D = rowsum(dO * O) (fp32, [hq, N]) and zeroes the fp32 dQ accumulator
+//   bwd_main    one CTA per (segment, 128-key tile n, kv-head g); loops over the
+//               G query heads of the group and the query tiles m >= n.  dK and
+//               dV of the tile accumulate in TMEM across the whole loop (GQA head
+//               sharing: the K/V tile is loaded once for all G heads); the dQ
+//               contribution of every (m, h) is added to the fp32 accumulator
+//               with vector reductions.
+//   bwd_dq_cvt  fp32 dQ accumulator -> bf16 dq
+//
+// bwd_main per (m, h), with the key rows of the tile on TMEM lanes:
+//   St  = K_n Q_m^T                 (TMEM cols [0,128))
+//   dPt = V_n dO_m^T                (TMEM cols [128,256))
+//   compute warps: Pt = exp2(St*scale*log2e - lse*log2e) (causal + validity mask),
+//                  dSt = scale * Pt * (dPt - D); both to shared memory as bf16
+//   dV += Pt dO_m, dK += dSt Q_m    (TMEM cols [256,256+D), [384,384+D))
+//   dQ  = dSt^T K_n                 (TMEM cols [0,D), reusing St)
+//   compute warps: dQ rows (query rows on TMEM lanes) -> red.global.add.v4.f32
+// Warp roles as in the forward: warp 0 TMA, warp 1 MMA, warps 4-11 compute
+// (two warpgroups, each owning half of the 128 query columns / D columns).
+#include <cfloat>
+#include <cstdint>
+
+#include "internal.h"
+#include "sm100.cuh"
+
+namespace vcs {
+namespace {
+
+using namespace dev;
+
+constexpr int kThreads = 384;
+constexpr int kPreThreads = 256;
+
+template <int D>
+struct Bwd {
+  static constexpr int BM = 128;                 // key rows of the tile
+  static constexpr int BN = 128;                 // query rows per iteration
+  static constexpr int KB = D / 64;
+  static constexpr int TILE = BM * D * 2;
+  static constexpr int BLOCK = BM * 128;
+  static constexpr int PTILE = BM * BN * 2;
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = TILE;
+  static constexpr int OFF_Q = 2 * TILE;
+  static constexpr int OFF_DO = 3 * TILE;
+  static constexpr int OFF_PT = 4 * TILE;
+  static constexpr int OFF_DST = OFF_PT + PTILE;
+  static constexpr int OFF_ROW = OFF_DST + PTILE;        // lse2[2][128], dvec[2][128] fp32
+  static constexpr int OFF_BAR = OFF_ROW + 4 * 128 * 4;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr int TM_ST = 0, TM_DPT = 128, TM_DV = 256, TM_DK = 384, TM_DQ = 0;
+  static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K (K-major) x Q^T (K-major)
+  static constexpr uint32_t IDESC_KV = idesc_bf16(128, D, 0, 1);    // Pt/dSt (K-major) x dO/Q (MN-major)
+  static constexpr uint32_t IDESC_DQ = idesc_bf16(128, D, 1, 1);    // dS (MN-major) x K (MN-major)
+};
+
+struct BwdBars {
+  uint64_t kv_full;
+  uint64_t qdo_full;
+  uint64_t qdo_empty;
+  uint64_t s_full;
+  uint64_t p_full;
+  uint64_t dq_full;
+  uint64_t dq_free;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+
+__device__ __forceinline__ void on_timeout(BwdBars* b, int32_t* status) {
+  set_status(status, VCS_ERR_DEVICE_TIMEOUT);
+  *reinterpret_cast<volatile int32_t*>(&b->abort) = 1;
+}
+__device__ __forceinline__ bool aborted(BwdBars* b) {
+  return *reinterpret_cast<volatile int32_t*>(&b->abort) != 0;
+}
+
+__device__ __forceinline__ void red_add_v4(float* p, float a, float b, float c, float d) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(p), "f"(a), "f"(b), "f"(c), "f"(d) : "memory");
+}
+
+// ------------------------------------------------------------------ bwd_pre
+// One 16-byte chunk (8 elements) per thread; D/8 consecutive threads share a row.
+template <int D>
+__global__ void __launch_bounds__(kPreThreads) bwd_pre(const __nv_bfloat16* __restrict__ o,
+                                                       const __nv_bfloat16* __restrict__ dout, int64_t rows,
+                                                       int32_t hq, int64_t num_tokens, float* __restrict__ dvec,
+                                                       float* __restrict__ dq_acc) {
+  constexpr int CPR = D / 8;  // chunks per row
+  const int64_t total = rows * CPR;
+  for (int64_t c = blockIdx.x * (int64_t)kPreThreads + threadIdx.x; c - threadIdx.x < total;
+       c += (int64_t)gridDim.x * kPreThreads) {
+    float acc = 0.f;
+    if (c < total) {
+      const uint4 a = __ldg(reinterpret_cast<const uint4*>(o) + c);
+      const uint4 b = __ldg(reinterpret_cast<const uint4*>(dout) + c);
+      const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+      const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 fa = __bfloat1622float2(pa[e]);
+        const float2 fb = __bfloat1622float2(pb[e]);
+        acc = fmaf(fa.x, fb.x, acc);
+        acc = fmaf(fa.y, fb.y, acc);
+      }
+      float4* z = reinterpret_cast<float4*>(dq_acc) + 2 * c;
+      z[0] = make_float4(0.f, 0.f, 0.f, 0.f);
+      z[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int off = CPR / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (c < total && (c % CPR) == 0) {
+      const int64_t row = c / CPR;           // row = token * hq + head
+      const int64_t tok = row / hq;
+      const int64_t h = row - tok * hq;
+      dvec[h * num_tokens + tok] = acc;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ bwd_dq_cvt
+__global__ void __launch_bounds__(256) bwd_dq_cvt(const float* __restrict__ acc, __nv_bfloat16* __restrict__ dq,
+                                                  int64_t n8) {
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < n8; c += (int64_t)gridDim.x * blockDim.x) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(acc) + 2 * c);
+    const float4 b = __ldg(reinterpret_cast<const float4*>(acc) + 2 * c + 1);
+    uint4 r;
+    r.x = pack_bf16(a.x, a.y);
+    r.y = pack_bf16(a.z, a.w);
+    r.z = pack_bf16(b.x, b.y);
+    r.w = pack_bf16(b.z, b.w);
+    reinterpret_cast<uint4*>(dq)[c] = r;
+  }
+}
+
+// ------------------------------------------------------------------ bwd_main
+template <int D>
+__device__ __forceinline__ void issue_st(uint32_t tmem_d, uint32_t a_addr, uint32_t b_addr) {
+  using C = Bwd<D>;
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint32_t off = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
+    tc_mma_ss(tmem_d, smem_desc(a_addr + off, 16, 1024), smem_desc(b_addr + off, 16, 1024), C::IDESC_S, kk > 0);
+  }
+}
+// D(tmem) (+)= A(128 x 128, K-major, K = query) x B(128 queries x D, MN-major)
+template <int D>
+__device__ __forceinline__ void issue_kv(uint32_t tmem_d, uint32_t a_addr, uint32_t b_addr, bool accumulate) {
+  using C = Bwd<D>;
+#pragma unroll
+  for (int kk = 0; kk < C::BN / 16; ++kk) {
+    const uint32_t aoff = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
+    tc_mma_ss(tmem_d, smem_desc(a_addr + aoff, 16, 1024), smem_desc(b_addr + kk * 2048, C::BLOCK, 1024),
+              C::IDESC_KV, (accumulate || kk > 0) ? 1u : 0u);
+  }
+}
+// dQ(tmem) = dS (128 queries x 128 keys, MN-major view of dSt) x K (128 keys x D, MN-major)
+template <int D>
+__device__ __forceinline__ void issue_dq(uint32_t tmem_d, uint32_t dst_addr, uint32_t k_addr) {
+  using C = Bwd<D>;
+#pragma unroll
+  for (int kk = 0; kk < C::BM / 16; ++kk) {
+    tc_mma_ss(tmem_d, smem_desc(dst_addr + kk * 2048, C::BLOCK, 1024), smem_desc(k_addr + kk * 2048, C::BLOCK, 1024),
+              C::IDESC_DQ, kk > 0);
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_main(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+             const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+             const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens, int32_t max_seqlen,
+             int32_t hq, int32_t hkv, int32_t ntiles, float scale, float scale_log2,
+             const float* __restrict__ lse, const float* __restrict__ dvec, float* __restrict__ dq_acc,
+             __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status) {
+  using C = Bwd<D>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  BwdBars* bars = reinterpret_cast<BwdBars*>(smem + C::OFF_BAR);
+  float* lse2_s = reinterpret_cast<float*>(smem + C::OFF_ROW);         // [2][128]
+  float* dvec_s = lse2_s + 2 * 128;                                    // [2][128]
+
+  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
+  const int seg = blockIdx.x / hkv;
+  const int g = blockIdx.x - seg * hkv;
+  const int n = blockIdx.y;  // key tile
+  const int start = cu_seqlens[seg];
+  const int end = cu_seqlens[seg + 1];
+  if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen ||
+      (seg == 0 && start != 0) || (seg == num_segments - 1 && end != num_tokens)) {
+    if (threadIdx.x == 0 && n == 0 && g == 0) set_status(status, VCS_ERR_DEVICE_CHECK);
+    return;
+  }
+  const int L = end - start;
+  const int nq = (L + C::BN - 1) / C::BN;
+  if (n >= nq) return;
+  const int G = hq / hkv;
+  const int per_head = nq - n;            // query tiles m = n .. nq-1
+  const int iters = G * per_head;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t sbase = smem_u32(smem);
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->kv_full, 1);
+    mbar_init(&bars->qdo_full, 1);
+    mbar_init(&bars->qdo_empty, 1);
+    mbar_init(&bars->s_full, 1);
+    mbar_init(&bars->p_full, 256);
+    mbar_init(&bars->dq_full, 1);
+    mbar_init(&bars->dq_free, 256);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      tma_prefetch_desc(&tm_do);
+      mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
+#pragma unroll
+      for (int kb = 0; kb < C::KB; ++kb) {
+        tma_load_3d(smem + C::OFF_K + kb * C::BLOCK, &tm_k, &bars->kv_full, kb * 64, g, start + n * C::BM);
+        tma_load_3d(smem + C::OFF_V + kb * C::BLOCK, &tm_v, &bars->kv_full, kb * 64, g, start + n * C::BM);
+      }
+      for (int it = 0; it < iters; ++it) {
+        const int h = g * G + it / per_head;
+        const int m = n + it % per_head;
+        if (it > 0 && !mbar_wait(&bars->qdo_empty, (it - 1) & 1)) {
+          on_timeout(bars, status);
+          break;
+        }
+        if (aborted(bars)) break;
+        mbar_arrive_expect_tx(&bars->qdo_full, 2 * C::TILE);
+#pragma unroll
+        for (int kb = 0; kb < C::KB; ++kb) {
+          tma_load_3d(smem + C::OFF_Q + kb * C::BLOCK, &tm_q, &bars->qdo_full, kb * 64, h, start + m * C::BN);
+          tma_load_3d(smem + C::OFF_DO + kb * C::BLOCK, &tm_do, &bars->qdo_full, kb * 64, h, start + m * C::BN);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(&bars->kv_full, 0);
+      tc_fence_after();
+      for (int it = 0; ok && it < iters; ++it) {
+        if (!mbar_wait(&bars->qdo_full, it & 1)) { ok = false; break; }
+        if (it > 0 && !mbar_wait(&bars->dq_free, (it - 1) & 1)) { ok = false; break; }
+        tc_fence_after();
+        issue_st<D>(tmem + C::TM_ST, sbase + C::OFF_K, sbase + C::OFF_Q);
+        issue_st<D>(tmem + C::TM_DPT, sbase + C::OFF_V, sbase + C::OFF_DO);
+        tc_commit(&bars->s_full);
+        if (!mbar_wait(&bars->p_full, it & 1)) { ok = false; break; }
+        tc_fence_after();
+        issue_kv<D>(tmem + C::TM_DV, sbase + C::OFF_PT, sbase + C::OFF_DO, it > 0);
+        issue_kv<D>(tmem + C::TM_DK, sbase + C::OFF_DST, sbase + C::OFF_Q, it > 0);
+        issue_dq<D>(tmem + C::TM_DQ, sbase + C::OFF_DST, sbase + C::OFF_K);
+        tc_commit(&bars->dq_full);
+        tc_commit(&bars->qdo_empty);
+        if (aborted(bars)) { ok = false; break; }
+      }
+      if (!ok) on_timeout(bars, status);
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ compute
+    const int wg = (warp - 4) >> 2;          // query-column half / D-column half
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;          // TMEM lane: key row (P phase) / query row (dQ phase)
+    const int tw = threadIdx.x - 128 - wg * 128;  // 0..127 within the warpgroup
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const int kpos = n * C::BM + r;
+    bool ok = true;
+    for (int it = 0; it < iters; ++it) {
+      const int h = g * G + it / per_head;
+      const int m = n + it % per_head;
+      const int buf = it & 1;
+      // per-query lse (log2 domain) and D of this warpgroup's 64 query columns
+      if (tw < 64) {
+        const int qi = wg * 64 + tw;
+        const int qpos = m * C::BN + qi;
+        float l2 = __int_as_float(0x7f800000);  // +inf: query outside the segment -> P = 0
+        float dd = 0.f;
+        if (qpos < L) {
+          l2 = lse[(size_t)h * num_tokens + start + qpos] * 1.4426950408889634f;
+          dd = dvec[(size_t)h * num_tokens + start + qpos];
+        }
+        lse2_s[buf * 128 + qi] = l2;
+        dvec_s[buf * 128 + qi] = dd;
+      }
+      named_bar_sync(1 + wg, 128);
+      if (!mbar_wait(&bars->s_full, it & 1)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t sv[64], pv[64];
+      tmem_ld_32x32b_x32(trow + C::TM_ST + wg * 64, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld_32x32b_x32(trow + C::TM_ST + wg * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tmem_ld_32x32b_x32(trow + C::TM_DPT + wg * 64, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
+      tmem_ld_32x32b_x32(trow + C::TM_DPT + wg * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
+      tmem_ld_wait();
+      reg_fence<64>(sv);
+      reg_fence<64>(pv);
+      const bool diag = (m == n);
+      const uint32_t pt_addr = sbase + C::OFF_PT + wg * C::BLOCK + r * 128;
+      const uint32_t ds_addr = sbase + C::OFF_DST + wg * C::BLOCK + r * 128;
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        uint32_t wp[4], wd[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          float pe[2], de[2];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int c = ch * 8 + e * 2 + u;          // column within this half
+            const int qi = wg * 64 + c;
+            const float l2 = lse2_s[buf * 128 + qi];
+            float p = ex2(fmaf(__uint_as_float(sv[c]), scale_log2, -l2));
+            if (diag && r > qi) p = 0.f;               // key after query
+            pe[u] = p;
+            de[u] = p * (__uint_as_float(pv[c]) - dvec_s[buf * 128 + qi]) * scale;
+          }
+          wp[e] = pack_bf16(pe[0], pe[1]);
+          wd[e] = pack_bf16(de[0], de[1]);
+        }
+        const uint32_t sw = (uint32_t)((ch ^ (r & 7)) << 4);
+        st_shared_v4(pt_addr + sw, wp[0], wp[1], wp[2], wp[3]);
+        st_shared_v4(ds_addr + sw, wd[0], wd[1], wd[2], wd[3]);
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&bars->p_full);
+      // dQ of this (m, h): query rows on TMEM lanes, this warpgroup's D/2 columns
+      if (!mbar_wait(&bars->dq_full, it & 1)) { ok = false; break; }
+      tc_fence_after();
+      const int qrow = m * C::BN + r;
+      float* dst = dq_acc + ((size_t)(start + qrow) * hq + h) * D + wg * (D / 2);
+#pragma unroll
+      for (int c = 0; c < D / 64; ++c) {
+        uint32_t q32[32];
+        tmem_ld_32x32b_x32(trow + C::TM_DQ + wg * (D / 2) + c * 32, q32);
+        tmem_ld_wait();
+        reg_fence<32>(q32);
+        if (qrow < L) {
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            red_add_v4(dst + c * 32 + e * 4, __uint_as_float(q32[e * 4]), __uint_as_float(q32[e * 4 + 1]),
+                       __uint_as_float(q32[e * 4 + 2]), __uint_as_float(q32[e * 4 + 3]));
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&bars->dq_free);
+      if (aborted(bars)) { ok = false; break; }
+    }
+    if (!ok) {
+      on_timeout(bars, status);
+    } else {
+      // dK, dV rows of the tile (key rows on TMEM lanes), this warpgroup's D/2 columns
+      const bool valid = kpos < L;
+      const size_t base = ((size_t)(start + kpos) * hkv + g) * D + wg * (D / 2);
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        const uint32_t col = (which == 0 ? C::TM_DK : C::TM_DV) + wg * (D / 2);
+        __nv_bfloat16* outp = (which == 0 ? dk : dv) + base;
+#pragma unroll
+        for (int c = 0; c < D / 64; ++c) {
+          uint32_t v32[32];
+          tmem_ld_32x32b_x32(trow + col + c * 32, v32);
+          tmem_ld_wait();
+          reg_fence<32>(v32);
+          if (valid) {
+            uint4* d4 = reinterpret_cast<uint4*>(outp + c * 32);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              uint4 pk;
+              pk.x = pack_bf16(__uint_as_float(v32[q * 8 + 0]), __uint_as_float(v32[q * 8 + 1]));
+              pk.y = pack_bf16(__uint_as_float(v32[q * 8 + 2]), __uint_as_float(v32[q * 8 + 3]));
+              pk.z = pack_bf16(__uint_as_float(v32[q * 8 + 4]), __uint_as_float(v32[q * 8 + 5]));
+              pk.w = pack_bf16(__uint_as_float(v32[q * 8 + 6]), __uint_as_float(v32[q * 8 + 7]));
+              d4[q] = pk;
+            }
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+template <int D>
+cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
+                         void* dv, void* ws, cudaStream_t st) {
+  using C = Bwd<D>;
+  char* w = static_cast<char*>(ws) + kWsHeader;
+  float* dvec = reinterpret_cast<float*>(w);
+  float* dq_acc = reinterpret_cast<float*>(w + align256((size_t)a.hq * a.num_tokens * 4));
+  const int64_t rows = a.num_tokens * a.hq;
+  {
+    const int64_t total = rows * (D / 8);
+    int64_t blocks = (total + kPreThreads - 1) / kPreThreads;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    bwd_pre<D><<<(unsigned)blocks, kPreThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(o),
+                                                         static_cast<const __nv_bfloat16*>(dout), rows, a.hq,
+                                                         a.num_tokens, dvec, dq_acc);
+  }
+  alignas(64) CUtensorMap tq, tk, tv, tdo;
+  if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
+      !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
+      !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128) ||
+      !encode_tma_3d_bf16(&tdo, dout, D, a.hq, a.num_tokens, 64, 128))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  if (e != cudaSuccess) return e;
+  const int ntiles = (a.max_seqlen + C::BM - 1) / C::BM;
+  if (ntiles > 0) {
+    const int64_t gx = (int64_t)a.num_segments * a.hkv;
+    if (gx > INT32_MAX || ntiles > 65535) return cudaErrorInvalidConfiguration;
+    dim3 grid((unsigned)gx, (unsigned)ntiles, 1);
+    bwd_main<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, tdo, a.cu_seqlens, a.num_segments,
+                                                 (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles, a.scale,
+                                                 a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
+                                                 static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
+                                                 a.status);
+  }
+  {
+    const int64_t n8 = rows * D / 8;
+    int64_t blocks = (n8 + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    if (n8 > 0) bwd_dq_cvt<<<(unsigned)blocks, 256, 0, st>>>(dq_acc, static_cast<__nv_bfloat16*>(dq), n8);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t attn_bwd_ws_bytes(const AttnArgs& a) {
+  if (a.num_tokens < 0 || a.hq <= 0 || a.d <= 0) return kWsHeader;
+  return kWsHeader + align256((size_t)a.hq * a.num_tokens * 4) + align256((size_t)a.num_tokens * a.hq * a.d * 4);
+}
+
+cudaError_t launch_attn_bwd(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
+                            void* dv, void* ws, cudaStream_t st) {
+  if (a.d == 64) return launch_bwd_d<64>(a, o, lse, dout, dq, dk, dv, ws, st);
+  return launch_bwd_d<128>(a, o, lse, dout, dq, dk, dv, ws, st);
+}
+
+}  // namespace vcs

@@ -1,0 +1,69 @@
+// internal.h - launchers shared between the C-ABI layer (api.cu) and the
+// kernel translation units.  Not part of the public interface.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "vcs.h"
+
+namespace vcs {
+
+// ---- segment builder (segments.cu) ----
+struct SegWorkspace {
+  int64_t* step_off;    // [num_steps+1] exclusive prefix of img+txt over all steps
+  int64_t* txt_pre;     // [num_steps+1] exclusive prefix of txt over all steps
+  int32_t* traj_nseg;   // [num_traj]
+  int64_t* traj_ntok;   // [num_traj]
+  int32_t* traj_maxlen; // [num_traj]
+  int64_t* seg_base;    // [num_traj+1]
+  int64_t* tok_base;    // [num_traj+1]
+  int64_t* seg_start;   // [num_steps+1] start of every segment in the packed buffer
+  int32_t* seg_full;    // [num_steps] global step of the first full (screenshot) step a_j
+  int32_t* seg_new;     // [num_steps] global step of the first new step s_j
+  int32_t* seg_last;    // [num_steps] global step of the last step e_j
+  int32_t* seg_first;   // [num_steps] global step of the trajectory's first step
+  int64_t* totals;      // [4]: num_segments, num_tokens, max_seqlen, status
+};
+size_t seg_workspace_bytes(int32_t num_traj, int64_t num_steps);
+SegWorkspace seg_workspace_carve(void* ws, int32_t num_traj, int64_t num_steps);
+
+cudaError_t launch_seg_plan(const int32_t* cu_steps, int32_t num_traj, int64_t num_steps, const int32_t* step_img,
+                            const int32_t* step_txt, int32_t window, int32_t keep, int64_t seg_capacity,
+                            int64_t tok_capacity, vcs_sizes* sizes, const SegWorkspace& w, cudaStream_t st);
+cudaError_t launch_seg_build(const int32_t* cu_steps, int32_t num_traj, int32_t window, int32_t keep,
+                             const int32_t* step_img, int32_t* cu_seqlens, int32_t* seg_traj, int32_t* tok_gather,
+                             int32_t* tok_src_step, int32_t* tok_pos, uint8_t* tok_loss_mask,
+                             const SegWorkspace& w, cudaStream_t st);
+
+// ---- gather (gather.cu) ----
+cudaError_t launch_gather(const void* src, int64_t traj_tokens, const int32_t* tok_gather, int64_t num_tokens,
+                          int64_t row_bytes, void* dst, int32_t* dev_status, cudaStream_t st);
+
+// ---- attention (attn_fwd.cu, attn_bwd.cu) ----
+struct AttnArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const int32_t* cu_seqlens;
+  int32_t num_segments;
+  int64_t num_tokens;
+  int32_t max_seqlen;
+  int32_t hq, hkv, d;
+  float scale;
+  int32_t* status;  // device status word (workspace header)
+};
+size_t attn_fwd_ws_bytes(const AttnArgs& a);
+cudaError_t launch_attn_fwd(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st);
+size_t attn_bwd_ws_bytes(const AttnArgs& a);
+cudaError_t launch_attn_bwd(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
+                            void* dv, void* ws, cudaStream_t st);
+
+// TMA descriptor encoding through the driver entry point (no libcuda link).
+bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d, uint64_t heads, uint64_t tokens,
+                        uint32_t box_d, uint32_t box_rows);
+
+constexpr size_t kWsHeader = 256;  // attention workspace header (status word first)
+
+}  // namespace vcs

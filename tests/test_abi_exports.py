@@ -1,0 +1,61 @@
+"""The C ABI library loads and exports every entry point include/vcs.h declares (CPU only)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+LIB = os.path.join(ROOT, "paper_2607_11185_gb300", "libvcs.so")
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "vcs.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(vcs_[a-z0-9_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(LIB):
+        from paper_2607_11185_gb300 import build
+        build.build()
+    return ctypes.CDLL(LIB)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_without_gpu(lib):
+    lib.vcs_status_string.restype = ctypes.c_char_p
+    for code in range(9):
+        s = lib.vcs_status_string(code).decode()
+        assert s.startswith("VCS_")
+    assert lib.vcs_status_string(99).decode() == "VCS_ERR_UNKNOWN"
+
+
+def test_host_side_argument_errors_without_gpu(lib):
+    # rejected before any CUDA call: null pointers, bad window, unsupported head_dim
+    f = lib.vcs_plan_segments
+    f.restype = ctypes.c_int32
+    f.argtypes = [ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
+                  ctypes.c_int32, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+    assert f(None, 1, 4, None, None, 2, 0, None, None, 0, None) == 1          # INVALID_ARG
+    assert f(8, 1, 4, 8, 8, 0, 0, 8, 256, 1 << 20, None) == 1                  # window 0
+    assert f(256, 1, 4, 256, 256, 2, 0, 256, 256, 1, None) == 8               # workspace too small
+    g = lib.vcs_attn_fwd
+    g.restype = ctypes.c_int32
+    g.argtypes = [ctypes.c_void_p] * 4 + [ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                          ctypes.c_int32, ctypes.c_int32, ctypes.c_float, ctypes.c_void_p,
+                                          ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+    assert g(256, 256, 256, 256, 1, 10, 10, 2, 1, 96, 0.0, 256, 256, 256, 4096, None) == 2   # d=96 unsupported
+    assert g(256, 256, 256, 256, 1, 10, 10, 3, 2, 64, 0.0, 256, 256, 256, 4096, None) == 2   # hq % hkv
+    assert g(None, 256, 256, 256, 1, 10, 10, 2, 1, 64, 0.0, 256, 256, 256, 4096, None) == 1
+    assert g(264, 256, 256, 256, 1, 10, 10, 2, 1, 64, 0.0, 256, 256, 256, 4096, None) == 1   # misaligned q
+    lib.vcs_attn_fwd_workspace_size.restype = ctypes.c_size_t
+    lib.vcs_attn_fwd_workspace_size.argtypes = [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 4
+    assert g(256, 256, 256, 256, 1, 10, 10, 2, 1, 64, 0.0, 256, 256, 256, 0, None) == 8      # no workspace

@@ -1,0 +1,148 @@
+"""GPU attention forward vs the fp64 oracle.
+
+Tolerances: O max-abs 2e-2 (bf16 inputs, fp32 accumulation, bf16 output);
+lse max-abs 2e-3 (fp32 score accumulation over d <= 128 bf16 products and
+the hardware exp2/log2, whose relative error is ~1e-6 on values |lse| < 100).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import attention as oatt
+from oracle import segments as oseg
+from paper_2607_11185_gb300 import workloads
+from tests.gpu_cases import cu_from_lengths, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+O_TOL = 2e-2
+LSE_TOL = 2e-3
+
+
+def run_fwd(q, k, v, cu):
+    from paper_2607_11185_gb300 import vcs
+    dcu = torch.from_numpy(np.asarray(cu, np.int32)).cuda()
+    lens = np.diff(cu)
+    return vcs.attn_fwd(q, k, v, dcu, int(lens.max()) if len(lens) else 0)
+
+
+def compare_full(q, k, v, cu, o, lse):
+    ro, rl = oatt.attn_fwd(q.cpu(), k.cpu(), v.cpu(), cu)
+    err_o = np.abs(o.float().cpu().numpy() - ro).max()
+    err_l = np.abs(lse.cpu().numpy() - rl).max()
+    assert err_o <= O_TOL, err_o
+    assert err_l <= LSE_TOL, err_l
+
+
+CASES = [
+    # (lengths, hq, hkv, d)
+    ([1, 127, 128, 129, 255, 256, 257, 300], 2, 1, 64),
+    ([1, 127, 128, 129, 255, 256, 257, 300], 2, 1, 128),
+    ([600, 1, 383, 513], 7, 1, 128),           # GQA 7:1, odd number of tiles
+    ([640, 129], 4, 4, 64),                    # MHA
+    ([1000], 6, 2, 128),
+]
+
+
+@pytest.mark.parametrize("lengths,hq,hkv,d", CASES)
+def test_small_shapes_full_oracle(lengths, hq, hkv, d):
+    cu = cu_from_lengths(lengths)
+    q, k, v, _ = workloads.draw_dense(11 + d + hq, int(cu[-1]), hq, hkv, d, device="cuda")
+    o, lse = run_fwd(q, k, v, cu)
+    compare_full(q, k, v, cu, o, lse)
+
+
+def test_tiny_workload_full_oracle():
+    w = workloads.WORKLOADS["tiny"]
+    cu_s, img, txt = workloads.draw_steps(w)
+    lay = oseg.build(cu_s, img, txt, w.window, w.keep)
+    qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
+    g = torch.from_numpy(lay["tok_gather"].astype(np.int64)).cuda()
+    q, k, v = qt[g], kt[g], vt[g]
+    o, lse = run_fwd(q, k, v, lay["cu_seqlens"])
+    compare_full(q, k, v, lay["cu_seqlens"], o, lse)
+
+
+def test_single_token_segments_copy_v():
+    cu = cu_from_lengths([1] * 40)
+    q, k, v, _ = workloads.draw_dense(5, 40, 4, 2, 128, device="cuda")
+    o, lse = run_fwd(q, k, v, cu)
+    ref_v = v.repeat_interleave(2, dim=1)
+    assert torch.equal(o, ref_v)     # softmax over one key is exactly 1
+    s = (q.float() * k.float().repeat_interleave(2, 1)).sum(-1).T / math.sqrt(128)
+    assert (lse - s).abs().max().item() < LSE_TOL
+
+
+def test_large_logits_stress_rescaling():
+    # scores of magnitude ~40 force mid-loop maximum raises in the online softmax
+    cu = cu_from_lengths([700, 333])
+    q, k, v, _ = workloads.draw_dense(21, int(cu[-1]), 2, 1, 128, device="cuda", scale=6.0)
+    o, lse = run_fwd(q, k, v, cu)
+    compare_full(q, k, v, cu, o, lse)
+
+
+def check_sampled(q, k, v, cu, o, lse, rng, n_seg=6, heads=None):
+    nseg = len(cu) - 1
+    lens = np.diff(cu)
+    segs = sorted({int(np.argmin(lens)), int(np.argmax(lens)), 0, nseg - 1,
+                   *[int(x) for x in rng.integers(0, nseg, size=n_seg)]})
+    hq = q.shape[1]
+    heads = heads if heads is not None else sorted({0, hq - 1, int(rng.integers(0, hq))})
+    worst = 0.0
+    for s in segs:
+        b, e = int(cu[s]), int(cu[s + 1])
+        if e == b:
+            continue
+        rows = sample_rows(e - b, rng)
+        ro, rl = oatt.rows_fwd(q, k, v, (b, e), heads, rows)
+        idx = torch.tensor([b + r for r in rows], device=q.device)
+        got_o = o[idx][:, heads].float().cpu().numpy()
+        got_l = lse[heads][:, idx].cpu().numpy()
+        eo = np.abs(got_o - ro).max()
+        el = np.abs(got_l - rl).max()
+        worst = max(worst, eo)
+        assert eo <= O_TOL, (s, eo)
+        assert el <= LSE_TOL, (s, el)
+    return worst
+
+
+@pytest.mark.parametrize("name", ["traj8_w3", "traj32_w3"])
+def test_workload_full_size_sampled_rows(name):
+    w = workloads.WORKLOADS[name]
+    cu_s, img, txt = workloads.draw_steps(w)
+    lay = oseg.build(cu_s, img, txt, w.window, w.keep)
+    qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
+    g = torch.from_numpy(lay["tok_gather"].astype(np.int64)).cuda()
+    q, k, v = qt[g], kt[g], vt[g]
+    del qt, kt, vt
+    o, lse = run_fwd(q, k, v, lay["cu_seqlens"])
+    check_sampled(q, k, v, lay["cu_seqlens"], o, lse, np.random.default_rng(3))
+
+
+def test_long_horizon_outliers_sampled_rows():
+    # 16 x 50 steps, W=8, 40/8 heads, 5% of K rows scaled by 8; four trajectories at a time
+    w = workloads.WORKLOADS["traj16x50_w8"]
+    cu_s, img, txt = workloads.draw_steps(w)
+    lay = oseg.build(cu_s, img, txt, w.window, w.keep)
+    qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
+    cu = lay["cu_seqlens"]
+    # first four trajectories' segments
+    nseg4 = int(np.searchsorted(lay["seg_traj"], 4))
+    ntok4 = int(cu[nseg4])
+    g = torch.from_numpy(lay["tok_gather"][:ntok4].astype(np.int64)).cuda()
+    q, k, v = qt[g], kt[g], vt[g]
+    del qt, kt, vt
+    o, lse = run_fwd(q, k, v, cu[: nseg4 + 1])
+    check_sampled(q, k, v, cu[: nseg4 + 1], o, lse, np.random.default_rng(5),
+                  n_seg=3, heads=[0, 17, 39])
+
+
+def test_inconsistent_cu_seqlens_reported():
+    from paper_2607_11185_gb300 import vcs
+    q, k, v, _ = workloads.draw_dense(1, 64, 2, 1, 64, device="cuda")
+    bad = torch.tensor([0, 40, 30, 64], dtype=torch.int32, device="cuda")
+    with pytest.raises(vcs.VcsError) as e:
+        vcs.attn_fwd(q, k, v, bad, 64)
+    assert e.value.status == 6
