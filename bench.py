@@ -1,0 +1,438 @@
+"""Benchmark of the Visual Context Segmentation hot path on one GB300.
+
+One step = the whole hot path over one batch of synthetic trajectories:
+segment layout (vcs_build_segments), Q/K/V gather (vcs_gather), causal
+segmented attention forward (vcs_attn_fwd) and backward (vcs_attn_bwd).
+Trajectories are processed in chunks that fit HBM; every chunk's work is
+inside the timed region.
+
+Default workload: 16 trajectories x 50 steps, 2,700 screenshot + 512
+response tokens per step, window W=8, 40 query / 8 key-value heads, head_dim
+128, bf16, 5% of key rows scaled by 8 (the long-horizon stress workload).
+
+The printed value is credited attention TFLOP/s: 12 * d * Hq * sum_s L_s(L_s+1)/2
+(forward 4, backward 8; the backward's recomputation of S is not credited)
+divided by the device time of the whole step.
+
+--impl reference times the CPU oracle (fp64 numpy) on a bounded sample of the
+same workload instead (the oracle is the only reference implementation of
+this path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2607_11185_gb300 import workloads  # noqa: E402
+
+METRIC = "segmented attn fwd+bwd TFLOP/s & % BF16 peak; segment tokens/s; vs CPU oracle"
+CHUNK_BYTES = 110 << 30   # per-chunk working set budget on the device
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), \
+            float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+def layout_stats(cu_steps, img, txt, window, keep):
+    """Host-side sizes of the layout from the closed form (input preparation only)."""
+    seg_lens, seg_traj = [], []
+    for b in range(len(cu_steps) - 1):
+        g0, g1 = int(cu_steps[b]), int(cu_steps[b + 1])
+        T = g1 - g0
+        if T == 0:
+            continue
+        ti, tx = img[g0:g1].astype(np.int64), txt[g0:g1].astype(np.int64)
+        s = 1
+        j = 0
+        while s <= T:
+            e = min(keep + window, T) if j == 0 else min(s + window - 1, T)
+            a = max(1, s - keep)
+            seg_lens.append(int(tx[: a - 1].sum() + ti[a - 1: e].sum() + tx[a - 1: e].sum()))
+            seg_traj.append(b)
+            s = e + 1
+            j += 1
+    return np.asarray(seg_lens, np.int64), np.asarray(seg_traj, np.int64)
+
+
+def credited_flops(seg_lens, hq, d):
+    pairs = (seg_lens * (seg_lens + 1) // 2).sum()
+    return 12.0 * d * hq * float(pairs), 4.0 * d * hq * float(pairs), 8.0 * d * hq * float(pairs)
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self):
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            idx = os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0"
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", idx, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.th = threading.Thread(target=self._read, daemon=True)
+            self.th.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 8:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[4 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+def make_chunks(seg_lens, seg_traj, num_traj, hq, hkv, d):
+    """Trajectory ranges whose per-chunk device buffers fit CHUNK_BYTES."""
+    per_tok = (2 * hq * d * 2 + 2 * hkv * d * 2) * 2 + hq * d * 4 + hq * 8 + 16
+    chunks, b0, acc = [], 0, 0
+    tok_per_traj = np.bincount(seg_traj, weights=seg_lens, minlength=num_traj).astype(np.int64)
+    for b in range(num_traj):
+        t = int(tok_per_traj[b]) * per_tok
+        if acc > 0 and acc + t > CHUNK_BYTES:
+            chunks.append((b0, b))
+            b0, acc = b, 0
+        acc += t
+    chunks.append((b0, num_traj))
+    return chunks
+
+
+class Path:
+    """Device-resident inputs and per-chunk buffers for the hot path."""
+
+    def __init__(self, w: workloads.Workload, window: int, keep: int, device):
+        from paper_2607_11185_gb300 import vcs
+        self.vcs = vcs
+        self.w, self.window, self.keep, self.dev = w, window, keep, device
+        cu, img, txt = workloads.draw_steps(w)
+        self.cu, self.img, self.txt = cu, img, txt
+        self.seg_lens, self.seg_traj = layout_stats(cu, img, txt, window, keep)
+        self.num_tokens = int(self.seg_lens.sum())
+        self.ntraj_tok = workloads.trajectory_tokens(img, txt)
+        step_off = np.concatenate([[0], np.cumsum(img.astype(np.int64) + txt)])
+        self.traj_tok_off = step_off[cu]
+        # resident inputs: step counts, trajectory Q/K/V, upstream gradient dO (segment layout)
+        self.q_traj, self.k_traj, self.v_traj = workloads.draw_traj_qkv(w, self.ntraj_tok, device=device)
+        self.dout = workloads.draw_dout(w, self.num_tokens, device=device)
+        self.chunks = make_chunks(self.seg_lens, self.seg_traj, w.num_traj, w.hq, w.hkv, w.d)
+        self.chunk_in = []
+        seg_cum = np.concatenate([[0], np.cumsum(self.seg_lens)])
+        max_tok = max_seg = max_steps = 0
+        for b0, b1 in self.chunks:
+            s0 = int(np.searchsorted(self.seg_traj, b0))
+            s1 = int(np.searchsorted(self.seg_traj, b1))
+            g0, g1 = int(cu[b0]), int(cu[b1])
+            ci = dict(b0=b0, b1=b1, s0=s0, s1=s1, tok0=int(seg_cum[s0]), tok1=int(seg_cum[s1]),
+                      cu=torch.from_numpy((cu[b0:b1 + 1] - cu[b0]).astype(np.int32)).to(device),
+                      img=torch.from_numpy(img[g0:g1].copy()).to(device),
+                      txt=torch.from_numpy(txt[g0:g1].copy()).to(device),
+                      ttok0=int(self.traj_tok_off[b0]), ttok1=int(self.traj_tok_off[b1]),
+                      nsteps=g1 - g0, max_seqlen=int(self.seg_lens[s0:s1].max()) if s1 > s0 else 0)
+            self.chunk_in.append(ci)
+            max_tok = max(max_tok, ci["tok1"] - ci["tok0"])
+            max_seg = max(max_seg, s1 - s0)
+            max_steps = max(max_steps, g1 - g0)
+        hq, hkv, d = w.hq, w.hkv, w.d
+        self.max_tok, self.max_seg = max_tok, max_seg
+        T = lambda *s, dt=torch.bfloat16: torch.empty(s, dtype=dt, device=device)  # noqa: E731
+        self.cu_seqlens = T(max_seg + 1, dt=torch.int32)
+        self.tok_gather = T(max_tok, dt=torch.int32)
+        self.tok_src = T(max_tok, dt=torch.int32)
+        self.tok_pos = T(max_tok, dt=torch.int32)
+        self.tok_mask = T(max_tok, dt=torch.uint8)
+        self.sizes = torch.zeros(3, dtype=torch.int64, device=device)
+        self.seg_ws_bytes = vcs.vcs_segments_workspace_size(max(b1 - b0 for b0, b1 in self.chunks), max_steps)
+        self.seg_ws = T(self.seg_ws_bytes, dt=torch.uint8)
+        self.q, self.k, self.v = T(max_tok, hq, d), T(max_tok, hkv, d), T(max_tok, hkv, d)
+        self.o, self.lse = T(max_tok, hq, d), T(hq, max_tok, dt=torch.float32)
+        self.dq, self.dk, self.dv = T(max_tok, hq, d), T(max_tok, hkv, d), T(max_tok, hkv, d)
+        self.gstatus = torch.zeros(1, dtype=torch.int32, device=device)
+        mxl = int(self.seg_lens.max())
+        self.fwd_ws_bytes = vcs.vcs_attn_fwd_workspace_size(max_seg, max_tok, mxl, hq, hkv, d)
+        self.bwd_ws_bytes = vcs.vcs_attn_bwd_workspace_size(max_seg, max_tok, mxl, hq, hkv, d)
+        self.fwd_ws = T(self.fwd_ws_bytes, dt=torch.uint8)
+        self.bwd_ws = T(self.bwd_ws_bytes, dt=torch.uint8)
+        self.launches_per_step = 0
+
+    def step(self, stream, ev=None):
+        """One pass of the hot path over all chunks; optional (fwd, bwd) event pairs appended to ev."""
+        vcs, w = self.vcs, self.w
+        hq, hkv, d = w.hq, w.hkv, w.d
+        launches = 0
+        for ci in self.chunk_in:
+            nseg, ntok = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"]
+            st = vcs.vcs_build_segments(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"],
+                                        self.window, self.keep, self.max_seg, self.max_tok, self.cu_seqlens, None,
+                                        self.tok_gather, self.tok_src, self.tok_pos, self.tok_mask, self.sizes,
+                                        self.seg_ws, self.seg_ws_bytes, stream)
+            launches += 5
+            assert st == 0, vcs.vcs_status_string(st)
+            # the attention launch shape depends on the layout sizes: read them (one sync per chunk)
+            sz = self.sizes.cpu()
+            assert int(sz[0]) == nseg and int(sz[1]) == ntok and (int(sz[2]) >> 32) == 0
+            qt = self.q_traj[ci["ttok0"]:ci["ttok1"]]
+            kt = self.k_traj[ci["ttok0"]:ci["ttok1"]]
+            vt = self.v_traj[ci["ttok0"]:ci["ttok1"]]
+            st = vcs.vcs_gather(qt, kt, vt, ci["ttok1"] - ci["ttok0"], self.tok_gather, ntok, hq, hkv, d, self.q,
+                                self.k, self.v, self.gstatus, stream)
+            launches += 3
+            assert st == 0
+            e0 = e1 = e2 = None
+            if ev is not None:
+                e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+                e0.record(stream)
+            st = vcs.vcs_attn_fwd(self.q, self.k, self.v, self.cu_seqlens, nseg, ntok, ci["max_seqlen"], hq, hkv,
+                                  d, 0.0, self.o, self.lse, self.fwd_ws, self.fwd_ws_bytes, stream)
+            launches += 1
+            assert st == 0
+            if ev is not None:
+                e1.record(stream)
+            dout = self.dout[ci["tok0"]:ci["tok1"]]
+            st = vcs.vcs_attn_bwd(self.q, self.k, self.v, self.o, self.lse, dout, self.cu_seqlens, nseg, ntok,
+                                  ci["max_seqlen"], hq, hkv, d, 0.0, self.dq, self.dk, self.dv, self.bwd_ws,
+                                  self.bwd_ws_bytes, stream)
+            launches += 3
+            assert st == 0
+            if ev is not None:
+                e2.record(stream)
+                ev.append((e0, e1, e2, ci))
+        self.launches_per_step = launches
+
+    def device_status(self):
+        return (int(self.gstatus.item()), int(self.fwd_ws[:4].view(torch.int32).item()),
+                int(self.bwd_ws[:4].view(torch.int32).item()))
+
+
+def oracle_sample(w, window, keep, seconds_hint=True):
+    """The CPU oracle on a bounded sample: the builder on the whole batch, plus attention
+    forward + backward of one query head over the shortest segment."""
+    from oracle import attention as oatt
+    from oracle import segments as oseg
+    cu, img, txt = workloads.draw_steps(w)
+    t0 = time.perf_counter()
+    lay = oseg.build(cu, img, txt, window, keep, method="closed")
+    t_build = time.perf_counter() - t0
+    lens = np.diff(lay["cu_seqlens"]).astype(np.int64)
+    s = int(np.argmin(lens))
+    L = int(lens[s])
+    gen = torch.Generator().manual_seed(w.seed + 77)
+    q = torch.randn((L, 1, w.d), generator=gen).to(torch.bfloat16)
+    k = torch.randn((L, 1, w.d), generator=gen).to(torch.bfloat16)
+    v = torch.randn((L, 1, w.d), generator=gen).to(torch.bfloat16)
+    do = torch.randn((L, 1, w.d), generator=gen).to(torch.bfloat16)
+    t0 = time.perf_counter()
+    oatt.attn_bwd(q, k, v, do, [0, L])          # computes the forward too
+    t_attn = time.perf_counter() - t0
+    flops = 12.0 * w.d * 1 * L * (L + 1) / 2
+    sample = (f"oracle builder over all {len(cu) - 1} trajectories ({t_build:.2f} s) + fp64 attention fwd+bwd of "
+              f"1 query head over the shortest segment (L={L}, {t_attn:.2f} s)")
+    return flops / (t_build + t_attn) / 1e12, sample, t_build + t_attn
+
+
+def run_reference(args, w, window, keep, rank, world):
+    if rank != 0:
+        return
+    vals = []
+    for i in range(args.warmup + args.steps):
+        tflops, sample, secs = oracle_sample(w, window, keep)
+        if i >= args.warmup:
+            vals.append((tflops, secs))
+    v = statistics.median(x[0] for x in vals)
+    secs = statistics.median(x[1] for x in vals)
+    cores = os.cpu_count()
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "window": window, "keep": keep, "hq": w.hq, "hkv": w.hkv, "d": w.d},
+            "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="traj16x50_w8", choices=list(workloads.WORKLOADS))
+    ap.add_argument("--layout", default=None, choices=[None, *workloads.COMPARISON_LAYOUTS],
+                    help="lay the traj32_w3 draw out as one of the comparison layouts")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    w = workloads.WORKLOADS[args.workload]
+    window, keep = w.window, w.keep
+    if args.layout is not None:
+        window, keep = workloads.COMPARISON_LAYOUTS[args.layout]
+
+    if args.impl == "reference":
+        run_reference(args, w, window, keep, rank, world)
+        return
+
+    if world > 1:
+        import torch.distributed as dist
+        local = int(os.environ.get("LOCAL_RANK", rank))
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    # the CPU baseline runs before any GPU work so that no process pool or
+    # thread state is shared with the CUDA context
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, sample, _ = oracle_sample(w, window, keep)
+        cpu = {"value": v, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle", "sample": sample}
+
+    path = Path(w, window, keep, dev)
+    stream = torch.cuda.current_stream()
+    flops, f_fwd, f_bwd = credited_flops(path.seg_lens, w.hq, w.d)
+    for _ in range(args.warmup):
+        path.step(stream.cuda_stream)
+    torch.cuda.synchronize()
+    st = path.device_status()
+    assert st == (0, 0, 0), f"device status {st}"
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    clocks = ClockSampler()
+    clocks.start()
+    ev = []
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        path.step(stream.cuda_stream, ev)
+    t1.record(stream)
+    barrier()
+    ck = clocks.stop()
+    ms = t0.elapsed_time(t1) / args.steps
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = float(tt.item())
+    fwd_ms = sum(a.elapsed_time(b) for a, b, c, _ in ev) / args.steps
+    bwd_ms = sum(b.elapsed_time(c) for a, b, c, _ in ev) / args.steps
+    bwd_launch_ms = statistics.mean(b.elapsed_time(c) for a, b, c, _ in ev)
+    bwd_launch_flops = f_bwd / len(path.chunk_in)
+
+    value = flops * world / (ms / 1e3) / 1e12
+    burst, sustained, hbm, src = peaks()
+
+    # end to end through the public API with host buffers: pinned host -> device copies of the
+    # step's inputs and a device -> host read of its result, inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(path, args, flops * world, stream)
+
+    ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "window": window, "keep": keep, "num_traj": w.num_traj, "hq": w.hq,
+                   "hkv": w.hkv, "d": w.d, "segments": int(len(path.seg_lens)), "segment_tokens": path.num_tokens,
+                   "max_seqlen": int(path.seg_lens.max()), "chunks": len(path.chunk_in),
+                   "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)"},
+        "attn_tflop_credited": flops / 1e12,
+        "attn_fwd_ms": fwd_ms, "attn_bwd_ms": bwd_ms,
+        "attn_fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "attn_bwd_tflops": f_bwd / (bwd_ms / 1e3) / 1e12,
+        "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,
+        "frac_of_bf16_burst": value / burst, "frac_of_bf16_sustained": value / sustained,
+        "flash_convention_tflops": value * 14.0 / 12.0,
+        "segment_tokens_per_s": path.num_tokens * world / (ms / 1e3),
+        "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
+                     "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s", "frac": ach_bwd / sustained,
+                     "peak_source": f"{src} bf16 sustained", "traffic": None},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": path.launches_per_step * args.steps,
+        "clocks": ck,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_e2e(path, args, flops, stream):
+    """Same metric with inputs staged from pinned host memory and results read back."""
+    host = {}
+    try:
+        host["q"] = path.q_traj.cpu().pin_memory()
+        host["k"] = path.k_traj.cpu().pin_memory()
+        host["v"] = path.v_traj.cpu().pin_memory()
+        host["do"] = path.dout.cpu().pin_memory()
+        res = torch.empty(path.w.hq * path.max_tok, dtype=torch.float32).pin_memory()
+    except RuntimeError as e:
+        return {"value": None, "unit": "TFLOP/s", "error": f"pinned staging failed: {e}"[:200]}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = 0
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        path.q_traj.copy_(host["q"], non_blocking=True)
+        path.k_traj.copy_(host["k"], non_blocking=True)
+        path.v_traj.copy_(host["v"], non_blocking=True)
+        path.dout.copy_(host["do"], non_blocking=True)
+        path.step(stream.cuda_stream)
+        # result read back: the last chunk's log-sum-exp (the loss-side statistic)
+        res.copy_(path.lse.view(-1)[: res.numel()], non_blocking=True)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    d2h = res.numel() * 4
+    ms = t0.elapsed_time(t1) / args.steps
+    return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+if __name__ == "__main__":
+    main()
