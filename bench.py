@@ -193,9 +193,10 @@ class Path:
         self.bwd_ws = T(self.bwd_ws_bytes, dt=torch.uint8)
         self.launches_per_step = 0
 
-    def step(self, stream, ev=None):
+    def step(self, tstream, ev=None):
         """One pass of the hot path over all chunks; optional (fwd, bwd) event pairs appended to ev."""
         vcs, w = self.vcs, self.w
+        stream = tstream.cuda_stream
         hq, hkv, d = w.hq, w.hkv, w.d
         launches = 0
         for ci in self.chunk_in:
@@ -219,13 +220,13 @@ class Path:
             e0 = e1 = e2 = None
             if ev is not None:
                 e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-                e0.record(stream)
+                e0.record(tstream)
             st = vcs.vcs_attn_fwd(self.q, self.k, self.v, self.cu_seqlens, nseg, ntok, ci["max_seqlen"], hq, hkv,
                                   d, 0.0, self.o, self.lse, self.fwd_ws, self.fwd_ws_bytes, stream)
             launches += 1
             assert st == 0
             if ev is not None:
-                e1.record(stream)
+                e1.record(tstream)
             dout = self.dout[ci["tok0"]:ci["tok1"]]
             st = vcs.vcs_attn_bwd(self.q, self.k, self.v, self.o, self.lse, dout, self.cu_seqlens, nseg, ntok,
                                   ci["max_seqlen"], hq, hkv, d, 0.0, self.dq, self.dk, self.dv, self.bwd_ws,
@@ -233,7 +234,7 @@ class Path:
             launches += 3
             assert st == 0
             if ev is not None:
-                e2.record(stream)
+                e2.record(tstream)
                 ev.append((e0, e1, e2, ci))
         self.launches_per_step = launches
 
@@ -330,7 +331,7 @@ def main():
     stream = torch.cuda.current_stream()
     flops, f_fwd, f_bwd = credited_flops(path.seg_lens, w.hq, w.d)
     for _ in range(args.warmup):
-        path.step(stream.cuda_stream)
+        path.step(stream)
     torch.cuda.synchronize()
     st = path.device_status()
     assert st == (0, 0, 0), f"device status {st}"
@@ -348,7 +349,7 @@ def main():
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     for _ in range(args.steps):
-        path.step(stream.cuda_stream, ev)
+        path.step(stream, ev)
     t1.record(stream)
     barrier()
     ck = clocks.stop()
@@ -403,13 +404,21 @@ def main():
 
 def run_e2e(path, args, flops, stream):
     """Same metric with inputs staged from pinned host memory and results read back."""
+    srcs = {"q": path.q_traj, "k": path.k_traj, "v": path.v_traj, "do": path.dout}
+    need = sum(t.numel() * t.element_size() for t in srcs.values())
+    try:
+        avail = int(next(l for l in open("/proc/meminfo") if l.startswith("MemAvailable")).split()[1]) * 1024
+    except Exception:
+        avail = 0
+    if need > 0.6 * avail:
+        return {"value": None, "unit": "TFLOP/s",
+                "error": f"pinned staging of {need / 2**30:.0f} GiB exceeds 60% of available host memory"}
     host = {}
     try:
-        host["q"] = path.q_traj.cpu().pin_memory()
-        host["k"] = path.k_traj.cpu().pin_memory()
-        host["v"] = path.v_traj.cpu().pin_memory()
-        host["do"] = path.dout.cpu().pin_memory()
-        res = torch.empty(path.w.hq * path.max_tok, dtype=torch.float32).pin_memory()
+        for name, t in srcs.items():
+            host[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            host[name].copy_(t)
+        res = torch.empty(path.w.hq * path.max_tok, dtype=torch.float32, pin_memory=True)
     except RuntimeError as e:
         return {"value": None, "unit": "TFLOP/s", "error": f"pinned staging failed: {e}"[:200]}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
@@ -423,7 +432,7 @@ def run_e2e(path, args, flops, stream):
         path.k_traj.copy_(host["k"], non_blocking=True)
         path.v_traj.copy_(host["v"], non_blocking=True)
         path.dout.copy_(host["do"], non_blocking=True)
-        path.step(stream.cuda_stream)
+        path.step(stream)
         # result read back: the last chunk's log-sum-exp (the loss-side statistic)
         res.copy_(path.lse.view(-1)[: res.numel()], non_blocking=True)
     t1.record(stream)
