@@ -171,6 +171,43 @@ vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void*
                         float softmax_scale, void* dq, void* dk, void* dv,
                         void* ws, size_t ws_bytes, void* stream);
 
+/* ------------------------------------------------------------------------ *
+ * Backward for callers that cannot allocate device memory.
+ *
+ * The paper has no counterpart to this call; it exists for users of this
+ * library.  vcs_attn_bwd needs a workspace from the caller.  Some callers
+ * cannot allocate one: a plugin whose host framework owns all device memory
+ * and passes it only the input and output tensors, or a latency-critical
+ * loop that must not call cudaMalloc (it can synchronise the device, and it
+ * can fail when memory is nearly full).  This variant computes exactly what
+ * vcs_attn_bwd computes (same arguments, layouts and errors, minus the
+ * workspace) but takes its workspace from a fixed array of
+ * VCS_NOALLOC_SCRATCH_BYTES compiled into the library, which every GPU that
+ * loads the library holds until the process exits.  Neither the caller nor
+ * the library allocates anything; the caller still passes all inputs and
+ * outputs.
+ *
+ *   dev_status  int32 device word or NULL: receives the device status word
+ *               (as the first int32 of vcs_attn_bwd's workspace would)
+ * Returns VCS_ERR_WORKSPACE, before any launch, when the problem needs more
+ * than VCS_NOALLOC_SCRATCH_BYTES (vcs_attn_bwd_workspace_size() tells the
+ * need: 256 + 4*hq*num_tokens + 4*num_tokens*hq*d bytes, each term rounded up
+ * to 256; e.g. hq = 28, d = 128 allows about 2,300 tokens).
+ * The first call on each device performs a one-time set-up (it looks up the
+ * array's device address); make that first call before any stream capture.
+ * Every call on a device shares the one array, which keeps the last call's
+ * contents (each call clears what must start at zero): calls that can overlap
+ * on the GPU (different streams without ordering between them) race on it and
+ * must not be issued.
+ * ------------------------------------------------------------------------ */
+#define VCS_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+vcs_status vcs_attn_bwd_noalloc(const void* q, const void* k, const void* v, const void* o, const float* lse,
+                                const void* dout, const int32_t* cu_seqlens, int32_t num_segments,
+                                int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
+                                float softmax_scale, void* dq, void* dk, void* dv, int32_t* dev_status,
+                                void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -57,9 +57,12 @@ _lib_bwd_ws = _sig("vcs_attn_bwd_workspace_size", _sz, [_i32, _i64, _i32, _i32, 
 _lib_bwd = _sig("vcs_attn_bwd", _i32,
                 [_p, _p, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p, _sz, _p])
 
+_lib_bwd_noalloc = _sig("vcs_attn_bwd_noalloc", _i32,
+                        [_p, _p, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p, _p])
+
 EXPORTED = ["vcs_status_string", "vcs_version", "vcs_segments_workspace_size", "vcs_plan_segments",
             "vcs_build_segments", "vcs_gather", "vcs_attn_fwd_workspace_size", "vcs_attn_fwd",
-            "vcs_attn_bwd_workspace_size", "vcs_attn_bwd"]
+            "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc"]
 
 LIB_PATH = _LIB_PATH
 
@@ -142,6 +145,22 @@ def vcs_attn_bwd(q, k, v, o, lse, dout, cu_seqlens, num_segments, num_tokens, ma
     return _lib_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout), _ptr(cu_seqlens), num_segments,
                     num_tokens, max_seqlen, hq, hkv, d, softmax_scale, _ptr(dq), _ptr(dk), _ptr(dv), _ptr(ws),
                     ws_bytes, _stream(stream))
+
+
+def vcs_attn_bwd_noalloc(q, k, v, o, lse, dout, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d,
+                         softmax_scale, dq, dk, dv, dev_status, stream=None) -> int:
+    """vcs_attn_bwd with the library's fixed scratch instead of a caller workspace.
+
+    For callers that cannot allocate device memory (see include/vcs.h): all
+    inputs and outputs are still the caller's; the problem must fit the fixed
+    scratch, else VCS_ERR_WORKSPACE is returned before any launch.
+    """
+    return _lib_bwd_noalloc(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout), _ptr(cu_seqlens),
+                            num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale, _ptr(dq), _ptr(dk),
+                            _ptr(dv), _ptr(dev_status), _stream(stream))
+
+
+NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 # ---------------------------------------------------------------- conveniences
