@@ -192,9 +192,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* dvec_s = lse2_s + 2 * 128;                                    // [2][128]
 
   if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
-  const int seg = blockIdx.x / hkv;
-  const int g = blockIdx.x - seg * hkv;
-  const int n = blockIdx.y;  // key tile
+  // x = key tile (fastest), so the CTAs resident at one time mostly belong to
+  // one (segment, kv-head) and their dQ reductions hit the same rows in L2
+  const int sg = (int)(blockIdx.z * 65535u + blockIdx.y);
+  if (sg >= num_segments * hkv) return;
+  const int seg = sg / hkv;
+  const int g = sg - seg * hkv;
+  const int n = blockIdx.x;  // key tile
   const int start = cu_seqlens[seg];
   const int end = cu_seqlens[seg + 1];
   if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen ||
@@ -293,23 +297,30 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const int kpos = n * C::BM + r;
     bool ok = true;
+    // per-query lse (log2 domain) and D of this warpgroup's 64 query columns,
+    // loaded one iteration ahead so the global-load latency is off the critical path
+    auto load_row_terms = [&](int it, float& l2, float& dd) {
+      const int h = g * G + it / per_head;
+      const int m = n + it % per_head;
+      const int qpos = m * C::BN + wg * 64 + tw;
+      l2 = __int_as_float(0x7f800000);  // +inf: query outside the segment -> P = 0
+      dd = 0.f;
+      if (tw < 64 && qpos < L) {
+        l2 = __ldg(&lse[(size_t)h * num_tokens + start + qpos]) * 1.4426950408889634f;
+        dd = __ldg(&dvec[(size_t)h * num_tokens + start + qpos]);
+      }
+    };
+    float next_l2, next_dd;
+    load_row_terms(0, next_l2, next_dd);
     for (int it = 0; it < iters; ++it) {
       const int h = g * G + it / per_head;
       const int m = n + it % per_head;
       const int buf = it & 1;
-      // per-query lse (log2 domain) and D of this warpgroup's 64 query columns
       if (tw < 64) {
-        const int qi = wg * 64 + tw;
-        const int qpos = m * C::BN + qi;
-        float l2 = __int_as_float(0x7f800000);  // +inf: query outside the segment -> P = 0
-        float dd = 0.f;
-        if (qpos < L) {
-          l2 = lse[(size_t)h * num_tokens + start + qpos] * 1.4426950408889634f;
-          dd = dvec[(size_t)h * num_tokens + start + qpos];
-        }
-        lse2_s[buf * 128 + qi] = l2;
-        dvec_s[buf * 128 + qi] = dd;
+        lse2_s[buf * 128 + wg * 64 + tw] = next_l2;
+        dvec_s[buf * 128 + wg * 64 + tw] = next_dd;
       }
+      if (it + 1 < iters) load_row_terms(it + 1, next_l2, next_dd);
       named_bar_sync(1 + wg, 128);
       if (!mbar_wait(&bars->s_full, it & 1)) { ok = false; break; }
       tc_fence_after();
@@ -355,21 +366,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const int qrow = m * C::BN + r;
       float* dst = dq_acc + ((size_t)(start + qrow) * hq + h) * D + wg * (D / 2);
+      // drain this warpgroup's dQ columns into registers, release TMEM, then reduce
+      uint32_t q32[D / 2];
 #pragma unroll
-      for (int c = 0; c < D / 64; ++c) {
-        uint32_t q32[32];
-        tmem_ld_32x32b_x32(trow + C::TM_DQ + wg * (D / 2) + c * 32, q32);
-        tmem_ld_wait();
-        reg_fence<32>(q32);
-        if (qrow < L) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            red_add_v4(dst + c * 32 + e * 4, __uint_as_float(q32[e * 4]), __uint_as_float(q32[e * 4 + 1]),
-                       __uint_as_float(q32[e * 4 + 2]), __uint_as_float(q32[e * 4 + 3]));
-        }
-      }
+      for (int c = 0; c < D / 64; ++c)
+        tmem_ld_32x32b_x32(trow + C::TM_DQ + wg * (D / 2) + c * 32,
+                           *reinterpret_cast<uint32_t(*)[32]>(&q32[c * 32]));
+      tmem_ld_wait();
+      reg_fence<D / 2>(q32);
       tc_fence_before();
       mbar_arrive(&bars->dq_free);
+      if (qrow < L) {
+#pragma unroll
+        for (int e = 0; e < D / 8; ++e)
+          red_add_v4(dst + e * 4, __uint_as_float(q32[e * 4]), __uint_as_float(q32[e * 4 + 1]),
+                     __uint_as_float(q32[e * 4 + 2]), __uint_as_float(q32[e * 4 + 3]));
+      }
       if (aborted(bars)) { ok = false; break; }
     }
     if (!ok) {
@@ -443,8 +455,8 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   const int ntiles = (a.max_seqlen + C::BM - 1) / C::BM;
   if (ntiles > 0) {
     const int64_t gx = (int64_t)a.num_segments * a.hkv;
-    if (gx > INT32_MAX || ntiles > 65535) return cudaErrorInvalidConfiguration;
-    dim3 grid((unsigned)gx, (unsigned)ntiles, 1);
+    if (gx > (int64_t)65535 * 65535) return cudaErrorInvalidConfiguration;
+    dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
     bwd_main<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, tdo, a.cu_seqlens, a.num_segments,
                                                  (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles, a.scale,
                                                  a.scale * 1.4426950408889634f, lse, dvec, dq_acc,

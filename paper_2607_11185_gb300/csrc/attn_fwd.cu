@@ -23,11 +23,15 @@
 // O0 [256,256+D), O1 [384,384+D).
 //
 // Per K/V tile j the MMA thread issues, in order,
-//   PV0(j): O0 += P0 V_j,  S0(j+1) = Q0 K_{j+1}^T,
-//   PV1(j): O1 += P1 V_j,  S1(j+1) = Q1 K_{j+1}^T,
-// so that the tensor pipe works on one tile while the softmax warps of the
-// other tile turn S into P (ping-pong).  P goes through shared memory in the
-// 128-byte-swizzled K-major layout the MMA reads.
+//   S0(j+1) = Q0 K_{j+1}^T  once softmax 0 has copied S0(j) to registers,
+//   S1(j+1) = Q1 K_{j+1}^T  likewise for tile 1,
+//   PV0(j):  O0 += P0(j) V_j once P0(j) is in shared memory,
+//   PV1(j):  O1 += P1(j) V_j,
+// so the next scores are computed while the softmax warps still work on the
+// current ones, and the two tiles keep the tensor pipe busy in turn.  P goes
+// through shared memory in the 128-byte-swizzled K-major layout the MMA
+// reads; a softmax warp computes its P in registers and only waits for the
+// previous P.V of its tile before storing it.
 //
 // Online softmax with a lazy running maximum: the row maximum used for P is
 // only raised (and O, l rescaled) when a new tile's maximum exceeds it by more
@@ -73,6 +77,7 @@ struct Bars {
   uint64_t kv_full[3];
   uint64_t kv_empty[3];
   uint64_t s_full[2];
+  uint64_t s_consumed[2];
   uint64_t p_full[2];
   uint64_t pv_done[2];
   uint32_t tmem_base;
@@ -149,6 +154,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->s_consumed[i], 128);
       mbar_init(&bars->p_full[i], 128);
       mbar_init(&bars->pv_done[i], 1);
     }
@@ -178,15 +184,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_3d(smem + C::OFF_Q1 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m1 * C::BM);
       }
       const uint64_t keep_l2 = l2_policy_evict_last();
+      // ring order K0, K1, V0, K2, V1, ..., K_{n-1}, V_{n-2}, V_{n-1}: keys run one
+      // tile ahead of values, since S(j+1) is issued before P(j).V_j
       for (int c = 0; c < 2 * nkv; ++c) {
-        const int j = c >> 1, slot = c % 3, round = c / 3;
+        const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
+        const int j = c == 2 * nkv - 1 ? nkv - 1 : (is_v ? (c - 2) >> 1 : (c + 1) >> 1);
+        const int slot = c % 3, round = c / 3;
         if (c >= 3 && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
           on_timeout(bars, status);
           break;
         }
         if (aborted(bars)) break;
         mbar_arrive_expect_tx(&bars->kv_full[slot], C::TILE);
-        const CUtensorMap* tm = (c & 1) ? &tm_v : &tm_k;
+        const CUtensorMap* tm = is_v ? &tm_v : &tm_k;
 #pragma unroll
         for (int kb = 0; kb < C::KB; ++kb)
           tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, &bars->kv_full[slot], kb * 64, g,
@@ -204,6 +214,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         addr = sbase + C::OFF_KV + slot * C::TILE;
         return true;
       };
+      // positions of K_j and V_j in the producer's ring order
+      auto k_item = [&](int j) { return j == 0 ? 0 : 2 * j - 1; };
+      auto v_item = [&](int j) { return j == nkv - 1 ? 2 * nkv - 1 : 2 * j + 2; };
       uint32_t kaddr = 0, vaddr = 0;
       if (ok) ok = acquire(0, kaddr);
       if (ok) {
@@ -217,32 +230,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (int j = 0; ok && j < nkv; ++j) {
         const bool next = j + 1 < nkv;
-        if (!acquire(2 * j + 1, vaddr)) { ok = false; break; }
-        if (next && !acquire(2 * j + 2, kaddr)) { ok = false; break; }
-        // tile 0
+        // S(j+1) of each tile as soon as its softmax has pulled S(j) out of TMEM
+        if (next) {
+          if (!acquire(k_item(j + 1), kaddr)) { ok = false; break; }
+          if (j + 1 <= m0) {
+            if (!mbar_wait(&bars->s_consumed[0], j & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
+            tc_commit(&bars->s_full[0]);
+          }
+          if (has1) {
+            if (!mbar_wait(&bars->s_consumed[1], j & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
+            tc_commit(&bars->s_full[1]);
+          }
+          tc_commit(&bars->kv_empty[k_item(j + 1) % 3]);
+        }
+        // then O += P(j) V_j as each tile's P arrives
+        if (!acquire(v_item(j), vaddr)) { ok = false; break; }
         if (j <= m0) {
           if (!mbar_wait(&bars->p_full[0], j & 1)) { ok = false; break; }
           tc_fence_after();
           issue_pv<D>(tmem + C::TM_O0, sbase + C::OFF_P0, vaddr, j > 0);
           tc_commit(&bars->pv_done[0]);
-          if (next && j + 1 <= m0) {
-            issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
-            tc_commit(&bars->s_full[0]);
-          }
         }
-        // tile 1
         if (has1) {
           if (!mbar_wait(&bars->p_full[1], j & 1)) { ok = false; break; }
           tc_fence_after();
           issue_pv<D>(tmem + C::TM_O1, sbase + C::OFF_P1, vaddr, j > 0);
           tc_commit(&bars->pv_done[1]);
-          if (next) {
-            issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
-            tc_commit(&bars->s_full[1]);
-          }
         }
-        tc_commit(&bars->kv_empty[(2 * j + 1) % 3]);
-        if (next) tc_commit(&bars->kv_empty[(2 * j + 2) % 3]);
+        tc_commit(&bars->kv_empty[v_item(j) % 3]);
         if (aborted(bars)) { ok = false; break; }
       }
       if (!ok) on_timeout(bars, status);
@@ -269,14 +288,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_32x32b_x32(trow + s_col + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&s[c * 32]));
         tmem_ld_wait();
         reg_fence<128>(s);
+        // S of this tile is in registers: the MMA may overwrite it with S(j+1)
+        tc_fence_before();
+        mbar_arrive(&bars->s_consumed[wg]);
         if (j == mt) {  // diagonal tile: key c is visible to row r iff c <= r
 #pragma unroll
           for (int c = 0; c < 128; ++c)
             if (c > r) s[c] = __float_as_uint(-FLT_MAX);
         }
-        float mx = -FLT_MAX;
+        // row maximum as a tree (8 independent partial maxima) to keep the chain short
+        float pm[8];
 #pragma unroll
-        for (int c = 0; c < 128; ++c) mx = fmaxf(mx, __uint_as_float(s[c]));
+        for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(s[u]);
+#pragma unroll
+        for (int c = 8; c < 128; c += 8)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) pm[u] = fmaxf(pm[u], __uint_as_float(s[c + u]));
+        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         const float mx2 = mx * scale_log2;
         float alpha = 1.f;
         bool rescale = false;
@@ -287,29 +316,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_run = mx2;
           rescale = true;
         }
+        // P in registers (bf16 pairs, packed over S) before waiting for the previous P.V
+        float rsp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial row sums
+#pragma unroll
+        for (int c2 = 0; c2 < 64; ++c2) {
+          const float p0 = ex2(fmaf(__uint_as_float(s[2 * c2]), scale_log2, -m_run));
+          const float p1 = ex2(fmaf(__uint_as_float(s[2 * c2 + 1]), scale_log2, -m_run));
+          rsp[c2 & 3] += p0 + p1;
+          s[c2] = pack_bf16(p0, p1);
+        }
         // the previous P.V of this tile must be done before P and O change
         if (j > 0) {
           if (!mbar_wait(&bars->pv_done[wg], (j - 1) & 1)) { ok = false; break; }
           tc_fence_after();
         }
-        float rs = 0.f;
 #pragma unroll
-        for (int kb = 0; kb < 2; ++kb) {
+        for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
           for (int ch = 0; ch < 8; ++ch) {
-            uint32_t w[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int c = kb * 64 + ch * 8 + e * 2;
-              const float p0 = ex2(fmaf(__uint_as_float(s[c]), scale_log2, -m_run));
-              const float p1 = ex2(fmaf(__uint_as_float(s[c + 1]), scale_log2, -m_run));
-              rs += p0 + p1;
-              w[e] = pack_bf16(p0, p1);
-            }
-            st_shared_v4(p_addr + kb * C::BLOCK + r * 128 + ((ch ^ (r & 7)) << 4), w[0], w[1], w[2], w[3]);
+            const int w0 = kb * 32 + ch * 4;
+            st_shared_v4(p_addr + kb * C::BLOCK + r * 128 + ((ch ^ (r & 7)) << 4), s[w0], s[w0 + 1], s[w0 + 2],
+                         s[w0 + 3]);
           }
-        }
-        l = l * alpha + rs;
+        l = l * alpha + ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3]));
         if (j > 0 && __any_sync(0xffffffffu, rescale)) {
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
