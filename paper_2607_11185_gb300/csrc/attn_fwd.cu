@@ -296,16 +296,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 128; ++c)
             if (c > r) s[c] = __float_as_uint(-FLT_MAX);
         }
-        // row maximum as a tree (8 independent partial maxima) to keep the chain short
+        // row maximum: 8 independent three-input chains (short dependency chains,
+        // two elements per instruction)
         float pm[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(s[u]);
+        for (int u = 0; u < 8; ++u) pm[u] = fmaxf(__uint_as_float(s[2 * u]), __uint_as_float(s[2 * u + 1]));
 #pragma unroll
-        for (int c = 8; c < 128; c += 8)
+        for (int c = 16; c < 128; c += 16)
 #pragma unroll
-          for (int u = 0; u < 8; ++u) pm[u] = fmaxf(pm[u], __uint_as_float(s[c + u]));
-        const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                               fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+          for (int u = 0; u < 8; ++u)
+            pm[u] = fmax3(pm[u], __uint_as_float(s[c + 2 * u]), __uint_as_float(s[c + 2 * u + 1]));
+        const float mx = fmax3(fmax3(pm[0], pm[1], pm[2]), fmax3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
         const float mx2 = mx * scale_log2;
         float alpha = 1.f;
         bool rescale = false;
@@ -316,14 +317,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_run = mx2;
           rescale = true;
         }
-        // P in registers (bf16 pairs, packed over S) before waiting for the previous P.V
-        float rsp[4] = {0.f, 0.f, 0.f, 0.f};  // independent partial row sums
+        // P in registers (bf16 pairs, packed over S) before waiting for the previous P.V;
+        // the scale-and-shift and the row sums run on packed fp32 pairs
+        const uint64_t sc2 = f2pack(scale_log2, scale_log2);
+        const uint64_t nm2 = f2pack(-m_run, -m_run);
+        uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial row sums
 #pragma unroll
         for (int c2 = 0; c2 < 64; ++c2) {
-          const float p0 = ex2(fmaf(__uint_as_float(s[2 * c2]), scale_log2, -m_run));
-          const float p1 = ex2(fmaf(__uint_as_float(s[2 * c2 + 1]), scale_log2, -m_run));
-          rsp[c2 & 3] += p0 + p1;
+          float x0, x1;
+          f2unpack(ffma2(f2pack(__uint_as_float(s[2 * c2]), __uint_as_float(s[2 * c2 + 1])), sc2, nm2), x0, x1);
+          const float p0 = ex2(x0), p1 = ex2(x1);
+          acc[c2 & 3] = fadd2(acc[c2 & 3], f2pack(p0, p1));
           s[c2] = pack_bf16(p0, p1);
+        }
+        float rsp[4];
+        {
+          float a0, a1, b0, b1;
+          f2unpack(fadd2(acc[0], acc[1]), a0, a1);
+          f2unpack(fadd2(acc[2], acc[3]), b0, b1);
+          rsp[0] = a0;
+          rsp[1] = a1;
+          rsp[2] = b0;
+          rsp[3] = b1;
         }
         // the previous P.V of this tile must be done before P and O change
         if (j > 0) {
