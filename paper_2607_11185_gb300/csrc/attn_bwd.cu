@@ -426,6 +426,358 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------ bwd_main_v2 (head_dim 128)
+// Same work unit and result as bwd_main, reorganised for overlap: the query
+// rows of every (query tile, head) are processed as 64-row sub-tiles that
+// alternate between two streams.  Each stream owns a compute warpgroup and its
+// own TMEM columns for S^T and dP^T, so while one stream's warpgroup turns
+// S^T/dP^T into P^T/dS^T (or drains its dQ), the tensor pipe works on the other
+// stream.  dQ^T = K^T dS^T (head dims on TMEM lanes) reuses the stream's S^T
+// columns and is reduced into the fp32 accumulator with coalesced scalar
+// reductions (32 consecutive head dims per warp instruction).
+//   TMEM: dV [0,128), dK [128,256), stream k: S^T [256+128k, +64), dP^T [+64, +128)
+//   smem: K, V (64 KB), 3-stage ring of Q/dO 64-row tiles (96 KB),
+//         P^T and dS^T per stream (64 KB), per-stream row terms (1 KB)
+struct V2 {
+  static constexpr int D = 128;
+  static constexpr int BM = 128;                 // key rows of the tile
+  static constexpr int BQ = 64;                  // query rows per sub-tile
+  static constexpr int NST = 3;                  // Q/dO ring stages
+  static constexpr int KVTILE = BM * D * 2;      // 32 KB
+  static constexpr int KVBLOCK = BM * 128;       // one 64-dim column block of K or V
+  static constexpr int QTILE = BQ * D * 2;       // 16 KB
+  static constexpr int QBLOCK = BQ * 128;        // one 64-dim column block of a Q/dO sub-tile
+  static constexpr int PT = BM * BQ * 2;         // 16 KB: 128 keys x 64 queries bf16
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = KVTILE;
+  static constexpr int OFF_Q = 2 * KVTILE;                     // stage s: Q at +s*2*QTILE, dO at +QTILE
+  static constexpr int OFF_PT = OFF_Q + NST * 2 * QTILE;       // stream k at +k*PT
+  static constexpr int OFF_DST = OFF_PT + 2 * PT;
+  static constexpr int OFF_ROW = OFF_DST + 2 * PT;             // stream k: -lse*log2e [64], -D*scale [64]
+  static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * BQ * 4;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr int TM_DV = 0, TM_DK = 128, TM_ST = 256;    // stream k: S^T at TM_ST + 128k, dP^T at +64
+  static constexpr uint32_t IDESC_S = idesc_bf16(128, BQ, 0, 0);   // K or V (K-major) x Q or dO^T (K-major)
+  static constexpr uint32_t IDESC_KV = idesc_bf16(128, D, 0, 1);   // P^T/dS^T (K-major) x dO/Q (MN-major)
+  static constexpr uint32_t IDESC_DQ = idesc_bf16(128, BQ, 1, 1);  // K^T (MN-major) x dS^T (MN-major)
+};
+static_assert(V2::SMEM <= 232448, "shared memory budget");
+
+struct V2Bars {
+  uint64_t kv_full;
+  uint64_t qdo_full[3];
+  uint64_t qdo_empty[3];
+  uint64_t s_full[2];
+  uint64_t p_full[2];
+  uint64_t dq_full[2];
+  uint64_t tmem_free[2];
+  uint64_t acc_done;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+
+__device__ __forceinline__ void red_add_f32(float* p, float v) {
+  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    bwd_main_v2(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens, int32_t max_seqlen,
+                int32_t hq, int32_t hkv, float scale, float scale_log2, const float* __restrict__ lse,
+                const float* __restrict__ dvec, float* __restrict__ dq_acc, __nv_bfloat16* __restrict__ dk,
+                __nv_bfloat16* __restrict__ dv, int32_t* status) {
+  using C = V2;
+  constexpr int D = C::D;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  V2Bars* bars = reinterpret_cast<V2Bars*>(smem + C::OFF_BAR);
+
+  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
+  const int sg = (int)(blockIdx.z * 65535u + blockIdx.y);
+  if (sg >= num_segments * hkv) return;
+  const int seg = sg / hkv;
+  const int g = sg - seg * hkv;
+  const int n = blockIdx.x;  // key tile
+  const int start = cu_seqlens[seg];
+  const int end = cu_seqlens[seg + 1];
+  if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen ||
+      (seg == 0 && start != 0) || (seg == num_segments - 1 && end != num_tokens)) {
+    if (threadIdx.x == 0 && n == 0 && g == 0) set_status(status, VCS_ERR_DEVICE_CHECK);
+    return;
+  }
+  const int L = end - start;
+  if (n * C::BM >= L) return;
+  const int G = hq / hkv;
+  const int nsub = (L - n * C::BM + C::BQ - 1) / C::BQ;  // 64-row query sub-tiles at or after this key tile
+  const int U = G * nsub;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t sbase = smem_u32(smem);
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bars->kv_full, 1);
+    for (int i = 0; i < 3; ++i) {
+      mbar_init(&bars->qdo_full[i], 1);
+      mbar_init(&bars->qdo_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->p_full[i], 128);
+      mbar_init(&bars->dq_full[i], 1);
+      mbar_init(&bars->tmem_free[i], 128);
+    }
+    mbar_init(&bars->acc_done, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_base;
+  auto abort_now = [&]() {
+    set_status(status, VCS_ERR_DEVICE_TIMEOUT);
+    *reinterpret_cast<volatile int32_t*>(&bars->abort) = 1;
+  };
+  auto aborted_now = [&]() { return *reinterpret_cast<volatile int32_t*>(&bars->abort) != 0; };
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      tma_prefetch_desc(&tm_do);
+      mbar_arrive_expect_tx(&bars->kv_full, 2 * C::KVTILE);
+#pragma unroll
+      for (int kb = 0; kb < 2; ++kb) {
+        tma_load_3d(smem + C::OFF_K + kb * C::KVBLOCK, &tm_k, &bars->kv_full, kb * 64, g, start + n * C::BM);
+        tma_load_3d(smem + C::OFF_V + kb * C::KVBLOCK, &tm_v, &bars->kv_full, kb * 64, g, start + n * C::BM);
+      }
+      for (int u = 0; u < U; ++u) {
+        const int h = g * G + u / nsub;
+        const int q0 = n * C::BM + (u % nsub) * C::BQ;
+        const int stage = u % 3;
+        if (u >= 3 && !mbar_wait(&bars->qdo_empty[stage], ((u / 3) - 1) & 1)) {
+          abort_now();
+          break;
+        }
+        if (aborted_now()) break;
+        mbar_arrive_expect_tx(&bars->qdo_full[stage], 2 * C::QTILE);
+        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::QTILE;
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb) {
+          tma_load_3d(qs + kb * C::QBLOCK, &tm_q, &bars->qdo_full[stage], kb * 64, h, start + q0);
+          tma_load_3d(qs + C::QTILE + kb * C::QBLOCK, &tm_do, &bars->qdo_full[stage], kb * 64, h, start + q0);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(&bars->kv_full, 0);
+      tc_fence_after();
+      const uint32_t kaddr = sbase + C::OFF_K, vaddr = sbase + C::OFF_V;
+      // S^T and dP^T of sub-tile u into its stream's columns
+      auto issue_s = [&](int u) -> bool {
+        const int k = u & 1, stage = u % 3;
+        if (!mbar_wait(&bars->qdo_full[stage], (u / 3) & 1)) return false;
+        if (u >= 2 && !mbar_wait(&bars->tmem_free[k], ((u >> 1) - 1) & 1)) return false;
+        tc_fence_after();
+        const uint32_t qa = sbase + C::OFF_Q + stage * 2 * C::QTILE, da = qa + C::QTILE;
+        const uint32_t st = tmem + C::TM_ST + 128 * k;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
+          const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
+          tc_mma_ss(st, smem_desc(kaddr + ko, 16, 1024), smem_desc(qa + qo, 16, 1024), C::IDESC_S, kk > 0);
+        }
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
+          const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
+          tc_mma_ss(st + 64, smem_desc(vaddr + ko, 16, 1024), smem_desc(da + qo, 16, 1024), C::IDESC_S, kk > 0);
+        }
+        tc_commit(&bars->s_full[k]);
+        return true;
+      };
+      // dV += P^T dO, dK += dS^T Q, dQ^T = K^T dS^T for sub-tile u
+      auto issue_kv = [&](int u) -> bool {
+        const int k = u & 1, stage = u % 3;
+        if (!mbar_wait(&bars->p_full[k], (u >> 1) & 1)) return false;
+        tc_fence_after();
+        const uint32_t qa = sbase + C::OFF_Q + stage * 2 * C::QTILE, da = qa + C::QTILE;
+        const uint32_t pt = sbase + C::OFF_PT + k * C::PT, ds = sbase + C::OFF_DST + k * C::PT;
+#pragma unroll
+        for (int kk = 0; kk < C::BQ / 16; ++kk)
+          tc_mma_ss(tmem + C::TM_DV, smem_desc(pt + kk * 32, 16, 1024), smem_desc(da + kk * 2048, C::QBLOCK, 1024),
+                    C::IDESC_KV, (u > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < C::BQ / 16; ++kk)
+          tc_mma_ss(tmem + C::TM_DK, smem_desc(ds + kk * 32, 16, 1024), smem_desc(qa + kk * 2048, C::QBLOCK, 1024),
+                    C::IDESC_KV, (u > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < C::BM / 16; ++kk)
+          tc_mma_ss(tmem + C::TM_ST + 128 * k, smem_desc(kaddr + kk * 2048, C::KVBLOCK, 1024),
+                    smem_desc(ds + kk * 2048, C::PT, 1024), C::IDESC_DQ, kk > 0 ? 1u : 0u);
+        tc_commit(&bars->dq_full[k]);
+        tc_commit(&bars->qdo_empty[stage]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      if (ok && U > 1) ok = issue_s(1);
+      for (int u = 0; ok && u < U; u += 2) {
+        if (!issue_kv(u)) { ok = false; break; }
+        if (u + 1 < U && !issue_kv(u + 1)) { ok = false; break; }
+        if (u + 2 < U && !issue_s(u + 2)) { ok = false; break; }
+        if (u + 3 < U && !issue_s(u + 3)) { ok = false; break; }
+        if (aborted_now()) { ok = false; break; }
+      }
+      tc_commit(&bars->acc_done);
+      if (!ok) abort_now();
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ compute
+    const int k = (warp - 4) >> 2;   // stream
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // TMEM lane: key row (P phase) / head dim (dQ phase)
+    const int tw = threadIdx.x - 128 - k * 128;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    const uint32_t st_col = C::TM_ST + 128 * k;
+    float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 2 * C::BQ;   // -lse*log2e per query
+    float* nds_s = nl2_s + C::BQ;                                                 // -D*scale per query
+    const uint32_t pt_row = sbase + C::OFF_PT + k * C::PT + r * 128;
+    const uint32_t ds_row = sbase + C::OFF_DST + k * C::PT + r * 128;
+    const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
+    auto row_terms = [&](int u, float& nl2, float& nds) {
+      nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
+      nds = 0.f;
+      if (u < U && tw < C::BQ) {
+        const int h = g * G + u / nsub;
+        const int q = n * C::BM + (u % nsub) * C::BQ + tw;
+        if (q < L) {
+          nl2 = -__ldg(&lse[(size_t)h * num_tokens + start + q]) * 1.4426950408889634f;
+          nds = -__ldg(&dvec[(size_t)h * num_tokens + start + q]) * scale;
+        }
+      }
+    };
+    float next_nl2, next_nds;
+    row_terms(k, next_nl2, next_nds);
+    bool ok = true;
+    for (int i = 0;; ++i) {
+      const int u = 2 * i + k;
+      if (u >= U) break;
+      const int h = g * G + u / nsub;
+      const int qoff = (u % nsub) * C::BQ;           // query offset from the key tile's first row
+      const int q0 = n * C::BM + qoff;               // first query (in-segment position)
+      if (tw < C::BQ) {
+        nl2_s[tw] = next_nl2;
+        nds_s[tw] = next_nds;
+      }
+      named_bar_sync(1 + k, 128);
+      row_terms(u + 2, next_nl2, next_nds);
+      if (!mbar_wait(&bars->s_full[k], i & 1)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t sv[64], pv[64];
+      tmem_ld_32x32b_x32(trow + st_col, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld_32x32b_x32(trow + st_col + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tmem_ld_32x32b_x32(trow + st_col + 64, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
+      tmem_ld_32x32b_x32(trow + st_col + 96, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
+      tmem_ld_wait();
+      reg_fence<64>(sv);
+      reg_fence<64>(pv);
+      const bool diag = qoff < C::BM;                // this sub-tile overlaps the key tile's rows
+#pragma unroll
+      for (int ch = 0; ch < 8; ++ch) {
+        uint32_t wp[4], wd[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int c = ch * 8 + e * 2;
+          const float2 nl = *reinterpret_cast<const float2*>(&nl2_s[c]);
+          const float2 nd = *reinterpret_cast<const float2*>(&nds_s[c]);
+          float x0, x1;
+          f2unpack(ffma2(f2pack(__uint_as_float(sv[c]), __uint_as_float(sv[c + 1])), sl2, f2pack(nl.x, nl.y)), x0, x1);
+          float p0 = ex2(x0), p1 = ex2(x1);
+          if (diag) {                                  // key after query: P = 0
+            if (r > qoff + c) p0 = 0.f;
+            if (r > qoff + c + 1) p1 = 0.f;
+          }
+          const uint64_t pp = f2pack(p0, p1);
+          const uint64_t t = ffma2(f2pack(__uint_as_float(pv[c]), __uint_as_float(pv[c + 1])), sc2, f2pack(nd.x, nd.y));
+          float d0, d1;
+          f2unpack(fmul2(pp, t), d0, d1);
+          wp[e] = pack_bf16(p0, p1);
+          wd[e] = pack_bf16(d0, d1);
+        }
+        const uint32_t sw = (uint32_t)((ch ^ (r & 7)) << 4);
+        st_shared_v4(pt_row + sw, wp[0], wp[1], wp[2], wp[3]);
+        st_shared_v4(ds_row + sw, wd[0], wd[1], wd[2], wd[3]);
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&bars->p_full[k]);
+      named_bar_sync(1 + k, 128);                      // everyone is done with this sub-tile's row terms
+      // dQ^T: head dim r on the TMEM lane, the sub-tile's 64 queries on the columns
+      if (!mbar_wait(&bars->dq_full[k], i & 1)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t qv[64];
+      tmem_ld_32x32b_x32(trow + st_col, *reinterpret_cast<uint32_t(*)[32]>(&qv[0]));
+      tmem_ld_32x32b_x32(trow + st_col + 32, *reinterpret_cast<uint32_t(*)[32]>(&qv[32]));
+      tmem_ld_wait();
+      reg_fence<64>(qv);
+      tc_fence_before();
+      mbar_arrive(&bars->tmem_free[k]);
+      float* dst = dq_acc + ((size_t)(start + q0) * hq + h) * D + r;
+      const int nq = min(C::BQ, L - q0);
+#pragma unroll
+      for (int c = 0; c < C::BQ; ++c)
+        if (c < nq) red_add_f32(dst + (size_t)c * hq * D, __uint_as_float(qv[c]));
+      if (aborted_now()) { ok = false; break; }
+    }
+    if (ok && !mbar_wait(&bars->acc_done, 0)) ok = false;
+    if (!ok) {
+      abort_now();
+    } else {
+      tc_fence_after();
+      // warpgroup 0 writes dK, warpgroup 1 writes dV (key row r on the TMEM lane)
+      const int kpos = n * C::BM + r;
+      const uint32_t col = k == 0 ? C::TM_DK : C::TM_DV;
+      __nv_bfloat16* outp = (k == 0 ? dk : dv) + ((size_t)(start + kpos) * hkv + g) * D;
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t v32[32];
+        tmem_ld_32x32b_x32(trow + col + c * 32, v32);
+        tmem_ld_wait();
+        reg_fence<32>(v32);
+        if (kpos < L) {
+          uint4* d4 = reinterpret_cast<uint4*>(outp + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint4 pk;
+            pk.x = pack_bf16(__uint_as_float(v32[q * 8 + 0]), __uint_as_float(v32[q * 8 + 1]));
+            pk.y = pack_bf16(__uint_as_float(v32[q * 8 + 2]), __uint_as_float(v32[q * 8 + 3]));
+            pk.z = pack_bf16(__uint_as_float(v32[q * 8 + 4]), __uint_as_float(v32[q * 8 + 5]));
+            pk.w = pack_bf16(__uint_as_float(v32[q * 8 + 6]), __uint_as_float(v32[q * 8 + 7]));
+            d4[q] = pk;
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 template <int D>
@@ -450,18 +802,32 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
       !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128) ||
       !encode_tma_3d_bf16(&tdo, dout, D, a.hq, a.num_tokens, 64, 128))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  if (e != cudaSuccess) return e;
   const int ntiles = (a.max_seqlen + C::BM - 1) / C::BM;
+  const int64_t gx = (int64_t)a.num_segments * a.hkv;
+  if (gx > (int64_t)65535 * 65535) return cudaErrorInvalidConfiguration;
+  dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
   if (ntiles > 0) {
-    const int64_t gx = (int64_t)a.num_segments * a.hkv;
-    if (gx > (int64_t)65535 * 65535) return cudaErrorInvalidConfiguration;
-    dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
-    bwd_main<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, tdo, a.cu_seqlens, a.num_segments,
-                                                 (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles, a.scale,
-                                                 a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
-                                                 static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
-                                                 a.status);
+    if (D == 128) {
+      alignas(64) CUtensorMap tq64, tdo64;  // 64-row query sub-tiles
+      if (!encode_tma_3d_bf16(&tq64, a.q, D, a.hq, a.num_tokens, 64, 64) ||
+          !encode_tma_3d_bf16(&tdo64, dout, D, a.hq, a.num_tokens, 64, 64))
+        return cudaErrorInvalidValue;
+      cudaError_t e = cudaFuncSetAttribute(bwd_main_v2, cudaFuncAttributeMaxDynamicSharedMemorySize, V2::SMEM);
+      if (e != cudaSuccess) return e;
+      bwd_main_v2<<<grid, kThreads, V2::SMEM, st>>>(tq64, tk, tv, tdo64, a.cu_seqlens, a.num_segments,
+                                                    (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, a.scale,
+                                                    a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
+                                                    static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
+                                                    a.status);
+    } else {
+      cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+      if (e != cudaSuccess) return e;
+      bwd_main<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, tdo, a.cu_seqlens, a.num_segments,
+                                                   (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles, a.scale,
+                                                   a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
+                                                   static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
+                                                   a.status);
+    }
   }
   {
     const int64_t n8 = rows * D / 8;
