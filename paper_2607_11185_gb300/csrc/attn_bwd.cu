@@ -433,11 +433,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 // own TMEM columns for S^T and dP^T, so while one stream's warpgroup turns
 // S^T/dP^T into P^T/dS^T (or drains its dQ), the tensor pipe works on the other
 // stream.  dQ^T = K^T dS^T (head dims on TMEM lanes) reuses the stream's S^T
-// columns and is reduced into the fp32 accumulator with coalesced scalar
-// reductions (32 consecutive head dims per warp instruction).
+// columns; the warpgroup stages it in shared memory (in its own P^T/dS^T
+// buffer, free once dQ^T is computed) and one TMA bulk reduce-add per
+// sub-tile adds the 64 x 128 fp32 block to the dQ accumulator in L2.  The MMA
+// thread issues whichever stream's next MMAs are ready (non-blocking polls).
 //   TMEM: dV [0,128), dK [128,256), stream k: S^T [256+128k, +64), dP^T [+64, +128)
 //   smem: K, V (64 KB), 3-stage ring of Q/dO 64-row tiles (96 KB),
-//         P^T and dS^T per stream (64 KB), per-stream row terms (1 KB)
+//         per stream P^T | dS^T, later the dQ^T staging block (64 KB), row terms (1 KB)
 struct V2 {
   static constexpr int D = 128;
   static constexpr int BM = 128;                 // key rows of the tile
@@ -451,9 +453,8 @@ struct V2 {
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = KVTILE;
   static constexpr int OFF_Q = 2 * KVTILE;                     // stage s: Q at +s*2*QTILE, dO at +QTILE
-  static constexpr int OFF_PT = OFF_Q + NST * 2 * QTILE;       // stream k at +k*PT
-  static constexpr int OFF_DST = OFF_PT + 2 * PT;
-  static constexpr int OFF_ROW = OFF_DST + 2 * PT;             // stream k: -lse*log2e [64], -D*scale [64]
+  static constexpr int OFF_PD = OFF_Q + NST * 2 * QTILE;       // stream k at +2k*PT: P^T, then dS^T
+  static constexpr int OFF_ROW = OFF_PD + 4 * PT;              // stream k: -lse*log2e [64], -D*scale [64]
   static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * BQ * 4;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static constexpr int TM_DV = 0, TM_DK = 128, TM_ST = 256;    // stream k: S^T at TM_ST + 128k, dP^T at +64
@@ -476,13 +477,30 @@ struct V2Bars {
   int32_t abort;
 };
 
-__device__ __forceinline__ void red_add_f32(float* p, float v) {
-  asm volatile("red.global.add.f32 [%0], %1;" ::"l"(p), "f"(v) : "memory");
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
 }
+// dst (global, tensor map) += src (shared) for one box, asynchronously (bulk group).
+__device__ __forceinline__ void tma_reduce_add_3d(const void* map, const void* src, int x, int y, int z) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(map),
+      "r"(smem_u32(src)), "r"(x), "r"(y), "r"(z)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_main_v2(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                const __grid_constant__ CUtensorMap tm_dq,
                 const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens, int32_t max_seqlen,
                 int32_t hq, int32_t hkv, float scale, float scale_log2, const float* __restrict__ lse,
                 const float* __restrict__ dvec, float* __restrict__ dq_acc, __nv_bfloat16* __restrict__ dk,
@@ -611,7 +629,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(&bars->p_full[k], (u >> 1) & 1)) return false;
         tc_fence_after();
         const uint32_t qa = sbase + C::OFF_Q + stage * 2 * C::QTILE, da = qa + C::QTILE;
-        const uint32_t pt = sbase + C::OFF_PT + k * C::PT, ds = sbase + C::OFF_DST + k * C::PT;
+        const uint32_t pt = sbase + C::OFF_PD + 2 * k * C::PT, ds = pt + C::PT;
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
           tc_mma_ss(tmem + C::TM_DV, smem_desc(pt + kk * 32, 16, 1024), smem_desc(da + kk * 2048, C::QBLOCK, 1024),
@@ -628,14 +646,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_commit(&bars->qdo_empty[stage]);
         return true;
       };
-      if (ok) ok = issue_s(0);
-      if (ok && U > 1) ok = issue_s(1);
-      for (int u = 0; ok && u < U; u += 2) {
-        if (!issue_kv(u)) { ok = false; break; }
-        if (u + 1 < U && !issue_kv(u + 1)) { ok = false; break; }
-        if (u + 2 < U && !issue_s(u + 2)) { ok = false; break; }
-        if (u + 3 < U && !issue_s(u + 3)) { ok = false; break; }
-        if (aborted_now()) { ok = false; break; }
+      // issue S(u) and KV(u) in order of u each, whichever is ready first:
+      //   S(u) needs Q/dO of u and the stream's TMEM columns back (dQ^T of u-2 drained)
+      //   KV(u) needs P^T/dS^T of u
+      int next_s = 0, next_kv = 0;
+      long long idle_since = clock64();
+      while (ok && next_kv < U) {
+        bool progress = false;
+        if (next_s < U && next_s <= next_kv + 1) {
+          const int u = next_s;
+          if (mbar_test(&bars->qdo_full[u % 3], (u / 3) & 1) &&
+              (u < 2 || mbar_test(&bars->tmem_free[u & 1], ((u >> 1) - 1) & 1))) {
+            ok = issue_s(u);
+            ++next_s;
+            progress = true;
+          }
+        }
+        if (ok && next_kv < next_s && mbar_test(&bars->p_full[next_kv & 1], (next_kv >> 1) & 1)) {
+          ok = issue_kv(next_kv);
+          ++next_kv;
+          progress = true;
+        }
+        if (progress) {
+          idle_since = clock64();
+        } else if (clock64() - idle_since > kWaitLimitCycles || aborted_now()) {
+          ok = false;
+        }
       }
       tc_commit(&bars->acc_done);
       if (!ok) abort_now();
@@ -650,8 +686,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t st_col = C::TM_ST + 128 * k;
     float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 2 * C::BQ;   // -lse*log2e per query
     float* nds_s = nl2_s + C::BQ;                                                 // -D*scale per query
-    const uint32_t pt_row = sbase + C::OFF_PT + k * C::PT + r * 128;
-    const uint32_t ds_row = sbase + C::OFF_DST + k * C::PT + r * 128;
+    uint8_t* stage_buf = smem + C::OFF_PD + 2 * k * C::PT;           // P^T | dS^T, later dQ^T staging
+    const uint32_t pt_row = smem_u32(stage_buf) + r * 128;
+    const uint32_t ds_row = pt_row + C::PT;
     const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
     auto row_terms = [&](int u, float& nl2, float& nds) {
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
@@ -674,6 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int h = g * G + u / nsub;
       const int qoff = (u % nsub) * C::BQ;           // query offset from the key tile's first row
       const int q0 = n * C::BM + qoff;               // first query (in-segment position)
+      if (tw == 0 && i > 0) bulk_wait_read();    // the staging block is read before P^T overwrites it
       if (tw < C::BQ) {
         nl2_s[tw] = next_nl2;
         nds_s[tw] = next_nds;
@@ -731,13 +769,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       reg_fence<64>(qv);
       tc_fence_before();
       mbar_arrive(&bars->tmem_free[k]);
-      float* dst = dq_acc + ((size_t)(start + q0) * hq + h) * D + r;
-      const int nq = min(C::BQ, L - q0);
+      // stage dQ^T as a [64 queries][128 dims] fp32 block (query rows past the
+      // segment end are exact zeros) and add it to the accumulator with one TMA op
+      float* stg = reinterpret_cast<float*>(stage_buf);
 #pragma unroll
-      for (int c = 0; c < C::BQ; ++c)
-        if (c < nq) red_add_f32(dst + (size_t)c * hq * D, __uint_as_float(qv[c]));
+      for (int c = 0; c < C::BQ; ++c) stg[c * D + r] = __uint_as_float(qv[c]);
+      fence_proxy_async_smem();
+      named_bar_sync(1 + k, 128);
+      if (tw == 0) {
+        tma_reduce_add_3d(&tm_dq, stg, 0, h, start + q0);
+        bulk_commit();
+      }
       if (aborted_now()) { ok = false; break; }
     }
+    if (tw == 0) bulk_wait_all();
     if (ok && !mbar_wait(&bars->acc_done, 0)) ok = false;
     if (!ok) {
       abort_now();
@@ -808,13 +853,14 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
   if (ntiles > 0) {
     if (D == 128) {
-      alignas(64) CUtensorMap tq64, tdo64;  // 64-row query sub-tiles
+      alignas(64) CUtensorMap tq64, tdo64, tdq;  // 64-row query sub-tiles; fp32 dQ accumulator
       if (!encode_tma_3d_bf16(&tq64, a.q, D, a.hq, a.num_tokens, 64, 64) ||
-          !encode_tma_3d_bf16(&tdo64, dout, D, a.hq, a.num_tokens, 64, 64))
+          !encode_tma_3d_bf16(&tdo64, dout, D, a.hq, a.num_tokens, 64, 64) ||
+          !encode_tma_3d_f32(&tdq, dq_acc, D, a.hq, a.num_tokens, D, 64))
         return cudaErrorInvalidValue;
       cudaError_t e = cudaFuncSetAttribute(bwd_main_v2, cudaFuncAttributeMaxDynamicSharedMemorySize, V2::SMEM);
       if (e != cudaSuccess) return e;
-      bwd_main_v2<<<grid, kThreads, V2::SMEM, st>>>(tq64, tk, tv, tdo64, a.cu_seqlens, a.num_segments,
+      bwd_main_v2<<<grid, kThreads, V2::SMEM, st>>>(tq64, tk, tv, tdo64, tdq, a.cu_seqlens, a.num_segments,
                                                     (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, a.scale,
                                                     a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
                                                     static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
