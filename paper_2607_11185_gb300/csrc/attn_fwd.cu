@@ -14,24 +14,23 @@
 // index in decreasing order, so the longest rows of work start first.
 //
 // Warp roles (384 threads):
-//   warp 0      TMA producer: Q0/Q1 once, then K0,V0,K1,V1,... into a 3-slot ring
+//   warp 0      TMA producer: Q0/Q1 once, then K and V tiles into a 5-slot ring
+//               (K runs one tile ahead of V: K0, K1, V0, K2, V1, ...)
 //   warp 1      TMEM allocator and single-thread tcgen05.mma issuer
 //   warps 2-3   idle (they keep the softmax warps on TMEM lane quadrants 0-3)
 //   warps 4-7   softmax + epilogue for tile 0 (thread = query row)
 //   warps 8-11  softmax + epilogue for tile 1
 // TMEM (512 columns x 128 lanes, fp32): S0 [0,128), S1 [128,256),
-// O0 [256,256+D), O1 [384,384+D).
+// O0 [256,256+D), O1 [384,384+D).  P_k (bf16, two per column) overwrites the
+// first 64 columns of S_k and is the A operand of O_k += P_k V read straight
+// from TMEM, so P never touches shared memory.
 //
-// Per K/V tile j the MMA thread issues, in order,
-//   S0(j+1) = Q0 K_{j+1}^T  once softmax 0 has copied S0(j) to registers,
-//   S1(j+1) = Q1 K_{j+1}^T  likewise for tile 1,
-//   PV0(j):  O0 += P0(j) V_j once P0(j) is in shared memory,
-//   PV1(j):  O1 += P1(j) V_j,
-// so the next scores are computed while the softmax warps still work on the
-// current ones, and the two tiles keep the tensor pipe busy in turn.  P goes
-// through shared memory in the 128-byte-swizzled K-major layout the MMA
-// reads; a softmax warp computes its P in registers and only waits for the
-// previous P.V of its tile before storing it.
+// Per K/V tile j the MMA thread issues, for each tile k once its P_k(j) is in
+// TMEM: O_k += P_k(j) V_j, then S_k(j+1) = Q_k K_{j+1}^T.  The tensor pipe
+// executes in order, so the completion of S_k(j+1) also means that P_k(j) has
+// been consumed and O_k is up to date, which is all the softmax warps wait
+// for.  The two tiles alternate, so one tile's MMAs run while the other
+// tile's softmax warps work.
 //
 // Online softmax with a lazy running maximum: the row maximum used for P is
 // only raised (and O, l rescaled) when a new tile's maximum exceeds it by more
@@ -58,28 +57,25 @@ struct Fwd {
   static constexpr int KB = D / 64;                 // 128-byte column blocks per row
   static constexpr int TILE = BM * D * 2;           // bytes of a 128 x D bf16 tile
   static constexpr int BLOCK = BM * 128;            // bytes of one 128 x 64 column block
-  static constexpr int PTILE = BM * BN * 2;         // bytes of a 128 x 128 bf16 P tile
-  static constexpr int NSLOT = 3;
+  static constexpr int NSLOT = 5;
   static constexpr int OFF_Q0 = 0;
   static constexpr int OFF_Q1 = TILE;
   static constexpr int OFF_KV = 2 * TILE;
-  static constexpr int OFF_P0 = OFF_KV + NSLOT * TILE;
-  static constexpr int OFF_P1 = OFF_P0 + PTILE;
-  static constexpr int OFF_BAR = OFF_P1 + PTILE;
+  static constexpr int OFF_BAR = OFF_KV + NSLOT * TILE;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static constexpr int TM_S0 = 0, TM_S1 = 128, TM_O0 = 256, TM_O1 = 384;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // Q (K-major) x K^T (K-major)
-  static constexpr uint32_t IDESC_PV = idesc_bf16(128, D, 0, 1);    // P (K-major) x V (MN-major)
+  static constexpr uint32_t IDESC_PV = idesc_bf16(128, D, 0, 1);    // P (TMEM) x V (MN-major)
 };
+static_assert(Fwd<128>::SMEM <= 232448, "shared memory budget");
 
 struct Bars {
   uint64_t q_full;
-  uint64_t kv_full[3];
-  uint64_t kv_empty[3];
+  uint64_t kv_full[5];
+  uint64_t kv_empty[5];
   uint64_t s_full[2];
-  uint64_t s_consumed[2];
   uint64_t p_full[2];
-  uint64_t pv_done[2];
+  uint64_t o_done[2];
   uint32_t tmem_base;
   int32_t abort;
 };
@@ -100,16 +96,14 @@ __device__ __forceinline__ void issue_s(uint32_t tmem_d, uint32_t q_addr, uint32
   }
 }
 
+// O (+)= P V with P (128 x 128 keys, bf16) in TMEM columns p_tmem .. p_tmem+63.
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_addr, uint32_t v_addr, bool accumulate) {
+__device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_tmem, uint32_t v_addr, bool accumulate) {
   using C = Fwd<D>;
 #pragma unroll
-  for (int kk = 0; kk < C::BN / 16; ++kk) {
-    const uint32_t aoff = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
-    const uint32_t boff = kk * 16 * 128;  // 16 key rows of 128 bytes
-    tc_mma_ss(tmem_d, smem_desc(p_addr + aoff, 16, 1024), smem_desc(v_addr + boff, C::BLOCK, 1024), C::IDESC_PV,
+  for (int kk = 0; kk < C::BN / 16; ++kk)
+    tc_mma_ts(tmem_d, p_tmem + kk * 8, smem_desc(v_addr + kk * 16 * 128, C::BLOCK, 1024), C::IDESC_PV,
               (accumulate || kk > 0) ? 1u : 0u);
-  }
 }
 
 template <int D>
@@ -148,15 +142,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&bars->q_full, 1);
-    for (int i = 0; i < 3; ++i) {
+    for (int i = 0; i < C::NSLOT; ++i) {
       mbar_init(&bars->kv_full[i], 1);
       mbar_init(&bars->kv_empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_consumed[i], 128);
       mbar_init(&bars->p_full[i], 128);
-      mbar_init(&bars->pv_done[i], 1);
+      mbar_init(&bars->o_done[i], 1);
     }
     bars->abort = 0;
     fence_mbar_init();
@@ -184,13 +177,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_3d(smem + C::OFF_Q1 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m1 * C::BM);
       }
       const uint64_t keep_l2 = l2_policy_evict_last();
-      // ring order K0, K1, V0, K2, V1, ..., K_{n-1}, V_{n-2}, V_{n-1}: keys run one
-      // tile ahead of values, since S(j+1) is issued before P(j).V_j
+      // ring order K0, K1, V0, K2, V1, ..., K_{n-1}, V_{n-2}, V_{n-1}
       for (int c = 0; c < 2 * nkv; ++c) {
         const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
         const int j = c == 2 * nkv - 1 ? nkv - 1 : (is_v ? (c - 2) >> 1 : (c + 1) >> 1);
-        const int slot = c % 3, round = c / 3;
-        if (c >= 3 && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
+        const int slot = c % C::NSLOT, round = c / C::NSLOT;
+        if (c >= C::NSLOT && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
           on_timeout(bars, status);
           break;
         }
@@ -208,8 +200,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       bool ok = mbar_wait(&bars->q_full, 0);
       auto acquire = [&](int c, uint32_t& addr) -> bool {
-        const int slot = c % 3;
-        if (!mbar_wait(&bars->kv_full[slot], (c / 3) & 1)) return false;
+        const int slot = c % C::NSLOT;
+        if (!mbar_wait(&bars->kv_full[slot], (c / C::NSLOT) & 1)) return false;
         tc_fence_after();
         addr = sbase + C::OFF_KV + slot * C::TILE;
         return true;
@@ -230,38 +222,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (int j = 0; ok && j < nkv; ++j) {
         const bool next = j + 1 < nkv;
-        // S(j+1) of each tile as soon as its softmax has pulled S(j) out of TMEM
-        if (next) {
-          if (!acquire(k_item(j + 1), kaddr)) { ok = false; break; }
-          if (j + 1 <= m0) {
-            if (!mbar_wait(&bars->s_consumed[0], j & 1)) { ok = false; break; }
-            tc_fence_after();
-            issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
-            tc_commit(&bars->s_full[0]);
-          }
-          if (has1) {
-            if (!mbar_wait(&bars->s_consumed[1], j & 1)) { ok = false; break; }
-            tc_fence_after();
-            issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
-            tc_commit(&bars->s_full[1]);
-          }
-          tc_commit(&bars->kv_empty[k_item(j + 1) % 3]);
-        }
-        // then O += P(j) V_j as each tile's P arrives
         if (!acquire(v_item(j), vaddr)) { ok = false; break; }
+        if (next && !acquire(k_item(j + 1), kaddr)) { ok = false; break; }
+        // tile 0: O0 += P0(j) V_j, then S0(j+1)
         if (j <= m0) {
           if (!mbar_wait(&bars->p_full[0], j & 1)) { ok = false; break; }
           tc_fence_after();
-          issue_pv<D>(tmem + C::TM_O0, sbase + C::OFF_P0, vaddr, j > 0);
-          tc_commit(&bars->pv_done[0]);
+          issue_pv<D>(tmem + C::TM_O0, tmem + C::TM_S0, vaddr, j > 0);
+          if (next && j + 1 <= m0) {
+            issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
+            tc_commit(&bars->s_full[0]);
+          } else {
+            tc_commit(&bars->o_done[0]);
+          }
         }
+        // tile 1
         if (has1) {
           if (!mbar_wait(&bars->p_full[1], j & 1)) { ok = false; break; }
           tc_fence_after();
-          issue_pv<D>(tmem + C::TM_O1, sbase + C::OFF_P1, vaddr, j > 0);
-          tc_commit(&bars->pv_done[1]);
+          issue_pv<D>(tmem + C::TM_O1, tmem + C::TM_S1, vaddr, j > 0);
+          if (next) {
+            issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
+            tc_commit(&bars->s_full[1]);
+          } else {
+            tc_commit(&bars->o_done[1]);
+          }
         }
-        tc_commit(&bars->kv_empty[v_item(j) % 3]);
+        if (next) tc_commit(&bars->kv_empty[k_item(j + 1) % C::NSLOT]);
+        tc_commit(&bars->kv_empty[v_item(j) % C::NSLOT]);
         if (aborted(bars)) { ok = false; break; }
       }
       if (!ok) on_timeout(bars, status);
@@ -276,10 +264,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
       const uint32_t s_col = wg == 0 ? C::TM_S0 : C::TM_S1;
       const uint32_t o_col = wg == 0 ? C::TM_O0 : C::TM_O1;
-      const uint32_t p_addr = sbase + (wg == 0 ? C::OFF_P0 : C::OFF_P1);
+      const uint64_t sc2 = f2pack(scale_log2, scale_log2);
       float m_run = -FLT_MAX, l = 0.f;
       bool ok = true;
       for (int j = 0; j <= mt; ++j) {
+        // S(j) complete also means P(j-1) was consumed and O holds P(j-1) V
         if (!mbar_wait(&bars->s_full[wg], j & 1)) { ok = false; break; }
         tc_fence_after();
         uint32_t s[128];
@@ -288,16 +277,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_32x32b_x32(trow + s_col + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&s[c * 32]));
         tmem_ld_wait();
         reg_fence<128>(s);
-        // S of this tile is in registers: the MMA may overwrite it with S(j+1)
-        tc_fence_before();
-        mbar_arrive(&bars->s_consumed[wg]);
         if (j == mt) {  // diagonal tile: key c is visible to row r iff c <= r
 #pragma unroll
           for (int c = 0; c < 128; ++c)
             if (c > r) s[c] = __float_as_uint(-FLT_MAX);
         }
-        // row maximum: 8 independent three-input chains (short dependency chains,
-        // two elements per instruction)
+        // row maximum: 8 independent three-input chains
         float pm[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) pm[u] = fmaxf(__uint_as_float(s[2 * u]), __uint_as_float(s[2 * u + 1]));
@@ -317,11 +302,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           m_run = mx2;
           rescale = true;
         }
-        // P in registers (bf16 pairs, packed over S) before waiting for the previous P.V;
-        // the scale-and-shift and the row sums run on packed fp32 pairs
-        const uint64_t sc2 = f2pack(scale_log2, scale_log2);
+        // P = exp2(s*scale*log2e - m) as bf16 pairs, packed over S; the
+        // scale-and-shift and the row sums run on packed fp32 pairs
         const uint64_t nm2 = f2pack(-m_run, -m_run);
-        uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};  // independent partial row sums
+        uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
         for (int c2 = 0; c2 < 64; ++c2) {
           float x0, x1;
@@ -330,31 +314,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           acc[c2 & 3] = fadd2(acc[c2 & 3], f2pack(p0, p1));
           s[c2] = pack_bf16(p0, p1);
         }
-        float rsp[4];
-        {
-          float a0, a1, b0, b1;
-          f2unpack(fadd2(acc[0], acc[1]), a0, a1);
-          f2unpack(fadd2(acc[2], acc[3]), b0, b1);
-          rsp[0] = a0;
-          rsp[1] = a1;
-          rsp[2] = b0;
-          rsp[3] = b1;
-        }
-        // the previous P.V of this tile must be done before P and O change
-        if (j > 0) {
-          if (!mbar_wait(&bars->pv_done[wg], (j - 1) & 1)) { ok = false; break; }
-          tc_fence_after();
-        }
-#pragma unroll
-        for (int kb = 0; kb < 2; ++kb)
-#pragma unroll
-          for (int ch = 0; ch < 8; ++ch) {
-            const int w0 = kb * 32 + ch * 4;
-            st_shared_v4(p_addr + kb * C::BLOCK + r * 128 + ((ch ^ (r & 7)) << 4), s[w0], s[w0 + 1], s[w0 + 2],
-                         s[w0 + 3]);
-          }
-        l = l * alpha + ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3]));
+        float a0, a1, b0, b1;
+        f2unpack(fadd2(acc[0], acc[1]), a0, a1);
+        f2unpack(fadd2(acc[2], acc[3]), b0, b1);
+        l = l * alpha + ((a0 + a1) + (b0 + b1));
+        // P over the first 64 columns of S (the MMA reads it from there)
+        tmem_st_32x32b_x32(trow + s_col, *reinterpret_cast<uint32_t(*)[32]>(&s[0]));
+        tmem_st_32x32b_x32(trow + s_col + 32, *reinterpret_cast<uint32_t(*)[32]>(&s[32]));
         if (j > 0 && __any_sync(0xffffffffu, rescale)) {
+          const uint64_t al2 = f2pack(alpha, alpha);
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
             uint32_t o[32];
@@ -362,17 +330,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld_wait();
             reg_fence<32>(o);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            for (int e = 0; e < 32; e += 2) {
+              float x0, x1;
+              f2unpack(fmul2(f2pack(__uint_as_float(o[e]), __uint_as_float(o[e + 1])), al2), x0, x1);
+              o[e] = __float_as_uint(x0);
+              o[e + 1] = __float_as_uint(x1);
+            }
             tmem_st_32x32b_x32(trow + o_col + c * 32, o);
           }
-          tmem_st_wait();
         }
-        fence_proxy_async_smem();
+        tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&bars->p_full[wg]);
         if (aborted(bars)) { ok = false; break; }
       }
-      if (ok && !mbar_wait(&bars->pv_done[wg], mt & 1)) ok = false;
+      if (ok && !mbar_wait(&bars->o_done[wg], 0)) ok = false;
       if (!ok) {
         on_timeout(bars, status);
       } else {
@@ -380,6 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row = mt * C::BM + r;
         const bool valid = row < L;
         const float inv_l = 1.f / l;
+        const uint64_t il2 = f2pack(inv_l, inv_l);
         __nv_bfloat16* orow = out + ((size_t)(start + row) * hq + h) * D;
 #pragma unroll
         for (int c = 0; c < D / 32; ++c) {
@@ -387,17 +360,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_32x32b_x32(trow + o_col + c * 32, o);
           tmem_ld_wait();
           reg_fence<32>(o);
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            float x0, x1;
+            f2unpack(fmul2(f2pack(__uint_as_float(o[2 * e]), __uint_as_float(o[2 * e + 1])), il2), x0, x1);
+            pk[e] = pack_bf16(x0, x1);
+          }
           if (valid) {
             uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
-            for (int v4 = 0; v4 < 4; ++v4) {
-              uint4 pk;
-              pk.x = pack_bf16(__uint_as_float(o[v4 * 8 + 0]) * inv_l, __uint_as_float(o[v4 * 8 + 1]) * inv_l);
-              pk.y = pack_bf16(__uint_as_float(o[v4 * 8 + 2]) * inv_l, __uint_as_float(o[v4 * 8 + 3]) * inv_l);
-              pk.z = pack_bf16(__uint_as_float(o[v4 * 8 + 4]) * inv_l, __uint_as_float(o[v4 * 8 + 5]) * inv_l);
-              pk.w = pack_bf16(__uint_as_float(o[v4 * 8 + 6]) * inv_l, __uint_as_float(o[v4 * 8 + 7]) * inv_l);
-              dst[v4] = pk;
-            }
+            for (int v4 = 0; v4 < 4; ++v4) dst[v4] = make_uint4(pk[4 * v4], pk[4 * v4 + 1], pk[4 * v4 + 2], pk[4 * v4 + 3]);
           }
         }
         if (valid) lse[(size_t)h * num_tokens + start + row] = (m_run + lg2(l)) * 0.69314718055994531f;

@@ -131,6 +131,18 @@ __device__ __forceinline__ void tc_mma_ss(uint32_t d_tmem, uint64_t adesc, uint6
       : "memory");
 }
 
+// D(tmem) (+)= A(tmem) * B(smem desc), kind::f16.  A is M rows on TMEM lanes
+// with two consecutive bf16 K-elements per 32-bit column (K = 16 per
+// instruction spans 8 columns).
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Shared-memory matrix descriptor (Blackwell format): start address, leading
 // and stride byte offsets (16-byte units), version 1 at bit 46, layout type
 // in bits 61..63 (2 = 128-byte swizzle).
