@@ -599,26 +599,33 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       bool ok = mbar_wait(&bars->kv_full, 0);
       tc_fence_after();
-      const uint32_t kaddr = sbase + C::OFF_K, vaddr = sbase + C::OFF_V;
+      // descriptors built once; the issue loops only add compile-time offsets
+      const uint64_t k_kmaj = smem_desc(sbase + C::OFF_K, 16, 1024);
+      const uint64_t v_kmaj = smem_desc(sbase + C::OFF_V, 16, 1024);
+      const uint64_t k_mnmaj = smem_desc(sbase + C::OFF_K, C::KVBLOCK, 1024);
+      const uint64_t q_kmaj = smem_desc(sbase + C::OFF_Q, 16, 1024);
+      const uint64_t q_mnmaj = smem_desc(sbase + C::OFF_Q, C::QBLOCK, 1024);
+      const uint64_t p_kmaj = smem_desc(sbase + C::OFF_PD, 16, 1024);
+      const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_PD + C::PT, C::PT, 1024);
       // S^T and dP^T of sub-tile u into its stream's columns
       auto issue_s = [&](int u) -> bool {
         const int k = u & 1, stage = u % 3;
         if (!mbar_wait(&bars->qdo_full[stage], (u / 3) & 1)) return false;
         if (u >= 2 && !mbar_wait(&bars->tmem_free[k], ((u >> 1) - 1) & 1)) return false;
         tc_fence_after();
-        const uint32_t qa = sbase + C::OFF_Q + stage * 2 * C::QTILE, da = qa + C::QTILE;
+        const uint64_t qd = desc_at(q_kmaj, stage * 2 * C::QTILE), dd = desc_at(qd, C::QTILE);
         const uint32_t st = tmem + C::TM_ST + 128 * k;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
           const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
-          tc_mma_ss(st, smem_desc(kaddr + ko, 16, 1024), smem_desc(qa + qo, 16, 1024), C::IDESC_S, kk > 0);
+          tc_mma_ss(st, desc_at(k_kmaj, ko), desc_at(qd, qo), C::IDESC_S, kk > 0);
         }
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
           const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
-          tc_mma_ss(st + 64, smem_desc(vaddr + ko, 16, 1024), smem_desc(da + qo, 16, 1024), C::IDESC_S, kk > 0);
+          tc_mma_ss(st + 64, desc_at(v_kmaj, ko), desc_at(dd, qo), C::IDESC_S, kk > 0);
         }
         tc_commit(&bars->s_full[k]);
         return true;
@@ -628,20 +635,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int k = u & 1, stage = u % 3;
         if (!mbar_wait(&bars->p_full[k], (u >> 1) & 1)) return false;
         tc_fence_after();
-        const uint32_t qa = sbase + C::OFF_Q + stage * 2 * C::QTILE, da = qa + C::QTILE;
-        const uint32_t pt = sbase + C::OFF_PD + 2 * k * C::PT, ds = pt + C::PT;
+        const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::QTILE), dmn = desc_at(qmn, C::QTILE);
+        const uint64_t pd = desc_at(p_kmaj, 2 * k * C::PT), sd = desc_at(pd, C::PT);
+        const uint64_t smn = desc_at(ds_mnmaj, 2 * k * C::PT);
+        const uint32_t acc0 = u > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DV, smem_desc(pt + kk * 32, 16, 1024), smem_desc(da + kk * 2048, C::QBLOCK, 1024),
-                    C::IDESC_KV, (u > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_ss(tmem + C::TM_DV, desc_at(pd, kk * 32), desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DK, smem_desc(ds + kk * 32, 16, 1024), smem_desc(qa + kk * 2048, C::QBLOCK, 1024),
-                    C::IDESC_KV, (u > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_ss(tmem + C::TM_DK, desc_at(sd, kk * 32), desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
 #pragma unroll
         for (int kk = 0; kk < C::BM / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_ST + 128 * k, smem_desc(kaddr + kk * 2048, C::KVBLOCK, 1024),
-                    smem_desc(ds + kk * 2048, C::PT, 1024), C::IDESC_DQ, kk > 0 ? 1u : 0u);
+          tc_mma_ss(tmem + C::TM_ST + 128 * k, desc_at(k_mnmaj, kk * 2048), desc_at(smn, kk * 2048), C::IDESC_DQ,
+                    kk > 0 ? 1u : 0u);
         tc_commit(&bars->dq_full[k]);
         tc_commit(&bars->qdo_empty[stage]);
         return true;

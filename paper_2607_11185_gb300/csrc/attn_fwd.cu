@@ -86,24 +86,26 @@ __device__ __forceinline__ void on_timeout(Bars* b, int32_t* status) {
 }
 __device__ __forceinline__ bool aborted(Bars* b) { return *reinterpret_cast<volatile int32_t*>(&b->abort) != 0; }
 
+// S = Q K^T; qd, kd are K-major descriptors of the Q tile and the K tile.
 template <int D>
-__device__ __forceinline__ void issue_s(uint32_t tmem_d, uint32_t q_addr, uint32_t k_addr) {
+__device__ __forceinline__ void issue_s(uint32_t tmem_d, uint64_t qd, uint64_t kd) {
   using C = Fwd<D>;
 #pragma unroll
   for (int kk = 0; kk < D / 16; ++kk) {
     const uint32_t off = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
-    tc_mma_ss(tmem_d, smem_desc(q_addr + off, 16, 1024), smem_desc(k_addr + off, 16, 1024), C::IDESC_S, kk > 0);
+    tc_mma_ss(tmem_d, desc_at(qd, off), desc_at(kd, off), C::IDESC_S, kk > 0);
   }
 }
 
-// O (+)= P V with P (128 x 128 keys, bf16) in TMEM columns p_tmem .. p_tmem+63.
+// O (+)= P V with P (128 x 128 keys, bf16) in TMEM columns p_tmem .. p_tmem+63;
+// vd is the MN-major descriptor of the V tile.
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_tmem, uint32_t v_addr, bool accumulate) {
+__device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_tmem, uint64_t vd, bool accumulate) {
   using C = Fwd<D>;
+  const uint32_t acc0 = accumulate ? 1u : 0u;
 #pragma unroll
   for (int kk = 0; kk < C::BN / 16; ++kk)
-    tc_mma_ts(tmem_d, p_tmem + kk * 8, smem_desc(v_addr + kk * 16 * 128, C::BLOCK, 1024), C::IDESC_PV,
-              (accumulate || kk > 0) ? 1u : 0u);
+    tc_mma_ts(tmem_d, p_tmem + kk * 8, desc_at(vd, kk * 16 * 128), C::IDESC_PV, kk > 0 ? 1u : acc0);
 }
 
 template <int D>
@@ -199,23 +201,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       bool ok = mbar_wait(&bars->q_full, 0);
-      auto acquire = [&](int c, uint32_t& addr) -> bool {
+      // descriptors built once; the issue loops only add compile-time offsets
+      const uint64_t q0d = smem_desc(sbase + C::OFF_Q0, 16, 1024), q1d = desc_at(q0d, C::TILE);
+      const uint64_t kv_kmaj = smem_desc(sbase + C::OFF_KV, 16, 1024);
+      const uint64_t kv_mnmaj = smem_desc(sbase + C::OFF_KV, C::BLOCK, 1024);
+      // wait for ring item c; returns the byte offset of its slot
+      auto acquire = [&](int c, uint32_t& slot_off) -> bool {
         const int slot = c % C::NSLOT;
         if (!mbar_wait(&bars->kv_full[slot], (c / C::NSLOT) & 1)) return false;
         tc_fence_after();
-        addr = sbase + C::OFF_KV + slot * C::TILE;
+        slot_off = slot * C::TILE;
         return true;
       };
       // positions of K_j and V_j in the producer's ring order
       auto k_item = [&](int j) { return j == 0 ? 0 : 2 * j - 1; };
       auto v_item = [&](int j) { return j == nkv - 1 ? 2 * nkv - 1 : 2 * j + 2; };
-      uint32_t kaddr = 0, vaddr = 0;
+      uint32_t kaddr = 0, vaddr = 0;  // slot byte offsets of K_{j+1} and V_j
       if (ok) ok = acquire(0, kaddr);
       if (ok) {
-        issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
+        issue_s<D>(tmem + C::TM_S0, q0d, desc_at(kv_kmaj, kaddr));
         tc_commit(&bars->s_full[0]);
         if (has1) {
-          issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
+          issue_s<D>(tmem + C::TM_S1, q1d, desc_at(kv_kmaj, kaddr));
           tc_commit(&bars->s_full[1]);
         }
         tc_commit(&bars->kv_empty[0]);
@@ -228,9 +235,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j <= m0) {
           if (!mbar_wait(&bars->p_full[0], j & 1)) { ok = false; break; }
           tc_fence_after();
-          issue_pv<D>(tmem + C::TM_O0, tmem + C::TM_S0, vaddr, j > 0);
+          issue_pv<D>(tmem + C::TM_O0, tmem + C::TM_S0, desc_at(kv_mnmaj, vaddr), j > 0);
           if (next && j + 1 <= m0) {
-            issue_s<D>(tmem + C::TM_S0, sbase + C::OFF_Q0, kaddr);
+            issue_s<D>(tmem + C::TM_S0, q0d, desc_at(kv_kmaj, kaddr));
             tc_commit(&bars->s_full[0]);
           } else {
             tc_commit(&bars->o_done[0]);
@@ -240,9 +247,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (has1) {
           if (!mbar_wait(&bars->p_full[1], j & 1)) { ok = false; break; }
           tc_fence_after();
-          issue_pv<D>(tmem + C::TM_O1, tmem + C::TM_S1, vaddr, j > 0);
+          issue_pv<D>(tmem + C::TM_O1, tmem + C::TM_S1, desc_at(kv_mnmaj, vaddr), j > 0);
           if (next) {
-            issue_s<D>(tmem + C::TM_S1, sbase + C::OFF_Q1, kaddr);
+            issue_s<D>(tmem + C::TM_S1, q1d, desc_at(kv_kmaj, kaddr));
             tc_commit(&bars->s_full[1]);
           } else {
             tc_commit(&bars->o_done[1]);

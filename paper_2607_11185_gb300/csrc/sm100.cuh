@@ -157,6 +157,13 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo_bytes
   return d;
 }
 
+// The same descriptor moved by `bytes` (a multiple of 16) within shared
+// memory: the start address is the low field in 16-byte units, so issue loops
+// build a descriptor once per buffer and add compile-time offsets (a single
+// thread issues every MMA, and building a descriptor from scratch per
+// instruction costs more than a narrow MMA takes to execute).
+__device__ __forceinline__ uint64_t desc_at(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
+
 // Instruction descriptor for kind::f16 with bf16 A/B and fp32 D.
 // a_mn / b_mn select MN-major operands (0 = K-major).
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_mn) {
