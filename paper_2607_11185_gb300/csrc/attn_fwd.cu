@@ -10,8 +10,10 @@
 // 128-row query tiles (m0 = 2p, m1 = 2p+1).  Both tiles stream the same K/V
 // tiles of kv-head h / (hq/hkv), so each K/V tile brought into shared memory
 // feeds 256 query rows.  Tiles above the diagonal are never visited; only the
-// diagonal tile is masked element-wise.  Grid: x = (segment, head), y = pair
-// index in decreasing order, so the longest rows of work start first.
+// diagonal tile is masked element-wise.  Grid: one dimension ordered by
+// (segment, kv-head, pair index from the last, query head in the group), so
+// the CTAs sharing a K/V stream run together and the longest pairs of each
+// stream start first.
 //
 // Warp roles (384 threads):
 //   warp 0      TMA producer: Q0/Q1 once, then K and V tiles into a 5-slot ring
@@ -122,9 +124,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   // once any CTA of this launch has given up on a wait, the rest stand down
   if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
-  const int seg = blockIdx.x / hq;
-  const int h = blockIdx.x - seg * hq;
-  const int p = npairs - 1 - (int)blockIdx.y;
+  // 1-D grid ordered (segment, kv-head, pair from the last, head in group):
+  // the CTAs that stream the same K/V tiles are launched together, so those
+  // tiles are read from HBM about once and then served from L2
+  const int G = hq / hkv;
+  int idx = (int)blockIdx.x;
+  const int hh = idx % G;
+  idx /= G;
+  const int p = npairs - 1 - idx % npairs;
+  idx /= npairs;
+  const int g = idx % hkv;
+  const int seg = idx / hkv;
+  const int h = g * G + hh;
   const int start = cu_seqlens[seg];
   const int end = cu_seqlens[seg + 1];
   if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen ||
@@ -137,7 +148,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int m0 = 2 * p, m1 = 2 * p + 1;
   const bool has1 = m1 * C::BM < L;
   const int nkv = has1 ? m1 + 1 : m0 + 1;
-  const int g = h / (hq / hkv);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = smem_u32(smem);
@@ -406,10 +416,10 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
   if (e != cudaSuccess) return e;
   const int npairs = (a.max_seqlen + 2 * C::BM - 1) / (2 * C::BM);
   if (npairs == 0) return cudaSuccess;
-  const int64_t gx = (int64_t)a.num_segments * a.hq;
-  if (gx > INT32_MAX || npairs > 65535) return cudaErrorInvalidConfiguration;
+  const int64_t gx = (int64_t)a.num_segments * a.hq * npairs;
+  if (gx > INT32_MAX) return cudaErrorInvalidConfiguration;
   const float scale_log2 = a.scale * 1.4426950408889634f;
-  dim3 grid((unsigned)gx, (unsigned)npairs, 1);
+  dim3 grid((unsigned)gx, 1, 1);
   attn_fwd_kernel<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens,
                                                      a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
                                                      static_cast<__nv_bfloat16*>(o), lse, a.status);
