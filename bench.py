@@ -53,6 +53,22 @@ def peaks():
         return 1900.0, 1700.0, 6800.0, "fallback"
 
 
+def measured_traffic(profile="attn_bwd_traj16x50_w8.md"):
+    """DRAM bytes per vcs_attn_bwd call from the committed ncu capture, or None when the
+    backward kernel sources changed since those counters were taken."""
+    import hashlib
+    try:
+        text = open(os.path.join(ROOT, "profiles", profile)).read()
+        vals = dict(line.split(": ", 1) for line in text.splitlines() if ": " in line and " " not in line.split(": ")[0])
+        src = b"".join(open(os.path.join(ROOT, "paper_2607_11185_gb300", "csrc", f), "rb").read()
+                       for f in ("attn_bwd.cu", "sm100.cuh"))
+        if hashlib.sha256(src).hexdigest()[:16] != vals["source_sha256_16"].strip():
+            return None
+        return int(vals["traffic_bytes_per_launch"])
+    except Exception:
+        return None
+
+
 def layout_stats(cu_steps, img, txt, window, keep):
     """Host-side sizes of the layout from the closed form (input preparation only)."""
     seg_lens, seg_traj = [], []
@@ -390,7 +406,9 @@ def main():
         "segment_tokens_per_s": path.num_tokens * world / (ms / 1e3),
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
                      "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s", "frac": ach_bwd / sustained,
-                     "peak_source": f"{src} bf16 sustained", "traffic": None},
+                     "peak_source": f"{src} bf16 sustained",
+                     "traffic": measured_traffic() if w.name == "traj16x50_w8" and (window, keep) == (w.window, w.keep)
+                     else None},
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": path.launches_per_step * args.steps,
