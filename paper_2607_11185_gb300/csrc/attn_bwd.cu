@@ -29,6 +29,9 @@
 //   compute warps: dQ rows (query rows on TMEM lanes) -> red.global.add.v4.f32
 // Warp roles as in the forward: warp 0 TMA, warp 1 MMA, warps 4-11 compute
 // (two warpgroups, each owning half of the 128 query columns / D columns).
+// For head_dim 128, bwd_main_d128 replaces bwd_main: 64-query sub-tiles in two
+// streams, P^T kept in TMEM, and a fourth warpgroup that drains dQ with TMA
+// bulk reduce-adds (described at the kernel).
 #include <cfloat>
 #include <cstdint>
 
@@ -426,25 +429,33 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// ------------------------------------------------------------------ bwd_main_v2 (head_dim 128)
-// Same work unit and result as bwd_main, reorganised for overlap: the query
-// rows of every (query tile, head) are processed as 64-row sub-tiles that
-// alternate between two streams.  Each stream owns a compute warpgroup and its
-// own TMEM columns for S^T and dP^T, so while one stream's warpgroup turns
-// S^T/dP^T into P^T/dS^T (or drains its dQ), the tensor pipe works on the other
-// stream.  dQ^T = K^T dS^T (head dims on TMEM lanes) reuses the stream's S^T
-// columns; the warpgroup stages it in shared memory (in its own P^T/dS^T
-// buffer, free once dQ^T is computed) and one TMA bulk reduce-add per
-// sub-tile adds the 64 x 128 fp32 block to the dQ accumulator in L2.  The MMA
-// thread issues whichever stream's next MMAs are ready (non-blocking polls).
-//   TMEM: dV [0,128), dK [128,256), stream k: S^T [256+128k, +64), dP^T [+64, +128)
-//   smem: K, V (64 KB), 3-stage ring of Q/dO 64-row tiles (96 KB),
-//         per stream P^T | dS^T, later the dQ^T staging block (64 KB), row terms (1 KB)
-struct V2 {
+// ------------------------------------------------------------------ bwd_main_d128 (head_dim 128)
+// Same work unit and result as bwd_main, reorganised for overlap.  The query
+// rows of every (query tile, head) are processed as 64-row sub-tiles; sub-tile
+// u belongs to stream u & 1.  Four warpgroups:
+//   WG0   warp 0: TMA producer (K and V once, Q/dO sub-tiles through a 3-stage ring)
+//         warp 1: TMEM allocation and the single MMA-issuing thread
+//   WG1/2 compute for stream 0/1: S^T, dP^T -> P^T (bf16, written back to TMEM
+//         over dP^T: the A operand of dV += P^T dO) and dS^T (bf16, shared
+//         memory: operand of dK += dS^T Q and dQ^T = K^T dS^T)
+//   WG3   dQ drain: takes dQ^T of each sub-tile (head dims on TMEM lanes, its 64
+//         queries on columns) as soon as its MMAs finish, hands the columns back
+//         to the stream, stages the block as [64 queries][128 dims] fp32 in shared
+//         memory and adds it to the fp32 dQ accumulator with one TMA bulk
+//         reduce-add (query rows past the segment end are exact zeros)
+// so that neither the compute warpgroups nor the tensor pipe wait for the
+// accumulation.  Registers are rebalanced per warpgroup with setmaxnreg
+// (80 / 176 / 176 / 80 per thread; the block launches with 128).
+//   TMEM: dV [0,128), dK [128,256),
+//         stream k: S^T, later dQ^T [256+128k, +64); dP^T, later P^T [+64, +128)
+//   smem: K, V (64 KB), 3-stage Q/dO ring (96 KB), dS^T per stream (32 KB), row terms (1 KB),
+//         dQ^T staging block (32 KB)
+struct D128 {
   static constexpr int D = 128;
   static constexpr int BM = 128;                 // key rows of the tile
   static constexpr int BQ = 64;                  // query rows per sub-tile
   static constexpr int NST = 3;                  // Q/dO ring stages
+  static constexpr int THREADS = 512;
   static constexpr int KVTILE = BM * D * 2;      // 32 KB
   static constexpr int KVBLOCK = BM * 128;       // one 64-dim column block of K or V
   static constexpr int QTILE = BQ * D * 2;       // 16 KB
@@ -453,18 +464,24 @@ struct V2 {
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = KVTILE;
   static constexpr int OFF_Q = 2 * KVTILE;                     // stage s: Q at +s*2*QTILE, dO at +QTILE
-  static constexpr int OFF_PD = OFF_Q + NST * 2 * QTILE;       // stream k at +2k*PT: P^T, then dS^T
-  static constexpr int OFF_ROW = OFF_PD + 4 * PT;              // stream k: -lse*log2e [64], -D*scale [64]
-  static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * BQ * 4;
+  static constexpr int OFF_DS = OFF_Q + NST * 2 * QTILE;       // stream k: dS^T at +k*PT
+  static constexpr int OFF_ROW = OFF_DS + 2 * PT;              // stream k: -lse*log2e [64], -D*scale [64]
+  static constexpr int OFF_STG = OFF_ROW + 2 * 2 * BQ * 4;
+  static constexpr int OFF_BAR = OFF_STG + BQ * D * 4;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static constexpr int TM_DV = 0, TM_DK = 128, TM_ST = 256;    // stream k: S^T at TM_ST + 128k, dP^T at +64
+  // registers per thread after rebalancing: WG0, each compute warpgroup, the drain warpgroup
+  static constexpr int REG_CTRL = 80, REG_COMPUTE = 176, REG_DRAIN = 80;
+  static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, BQ, 0, 0);   // K or V (K-major) x Q or dO^T (K-major)
-  static constexpr uint32_t IDESC_KV = idesc_bf16(128, D, 0, 1);   // P^T/dS^T (K-major) x dO/Q (MN-major)
+  static constexpr uint32_t IDESC_KV = idesc_bf16(128, D, 0, 1);   // P^T/dS^T (TMEM or K-major) x dO/Q (MN-major)
   static constexpr uint32_t IDESC_DQ = idesc_bf16(128, BQ, 1, 1);  // K^T (MN-major) x dS^T (MN-major)
 };
-static_assert(V2::SMEM <= 232448, "shared memory budget");
+static_assert(D128::SMEM <= 232448, "shared memory budget");
+static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D128::REG_LAUNCH,
+              "setmaxnreg targets exceed the registers the block is launched with");
 
-struct V2Bars {
+struct D128Bars {
   uint64_t kv_full;
   uint64_t qdo_full[3];
   uint64_t qdo_empty[3];
@@ -486,7 +503,7 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// dst (global, tensor map) += src (shared) for one box, asynchronously (bulk group).
+
 __device__ __forceinline__ void tma_reduce_add_3d(const void* map, const void* src, int x, int y, int z) {
   asm volatile(
       "cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(map),
@@ -497,19 +514,18 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-__global__ void __launch_bounds__(kThreads, 1)
-    bwd_main_v2(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                const __grid_constant__ CUtensorMap tm_dq,
-                const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens, int32_t max_seqlen,
-                int32_t hq, int32_t hkv, float scale, float scale_log2, const float* __restrict__ lse,
-                const float* __restrict__ dvec, float* __restrict__ dq_acc, __nv_bfloat16* __restrict__ dk,
-                __nv_bfloat16* __restrict__ dv, int32_t* status) {
-  using C = V2;
+__global__ void __launch_bounds__(D128::THREADS, 1)
+    bwd_main_d128(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                  const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+                  const __grid_constant__ CUtensorMap tm_dq, const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens,
+                  int32_t max_seqlen, int32_t hq, int32_t hkv, float scale, float scale_log2,
+                  const float* __restrict__ lse, const float* __restrict__ dvec, float* __restrict__ dq_acc,
+                  __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status) {
+  using C = D128;
   constexpr int D = C::D;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  V2Bars* bars = reinterpret_cast<V2Bars*>(smem + C::OFF_BAR);
+  D128Bars* bars = reinterpret_cast<D128Bars*>(smem + C::OFF_BAR);
 
   if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
   const int sg = (int)(blockIdx.z * 65535u + blockIdx.y);
@@ -563,9 +579,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   };
   auto aborted_now = [&]() { return *reinterpret_cast<volatile int32_t*>(&bars->abort) != 0; };
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    if (lane == 0) {
+  if (warp < 4) {
+    setmaxnreg_dec<C::REG_CTRL>();
+    if (warp == 0 && lane == 0) {
+      // ---------------------------------------------------------- producer
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
@@ -593,10 +610,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_3d(qs + C::QTILE + kb * C::QBLOCK, &tm_do, &bars->qdo_full[stage], kb * 64, h, start + q0);
         }
       }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    } else if (warp == 1 && lane == 0) {
+      // ---------------------------------------------------------- MMA issuer
       bool ok = mbar_wait(&bars->kv_full, 0);
       tc_fence_after();
       // descriptors built once; the issue loops only add compile-time offsets
@@ -605,13 +620,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t k_mnmaj = smem_desc(sbase + C::OFF_K, C::KVBLOCK, 1024);
       const uint64_t q_kmaj = smem_desc(sbase + C::OFF_Q, 16, 1024);
       const uint64_t q_mnmaj = smem_desc(sbase + C::OFF_Q, C::QBLOCK, 1024);
-      const uint64_t p_kmaj = smem_desc(sbase + C::OFF_PD, 16, 1024);
-      const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_PD + C::PT, C::PT, 1024);
+      const uint64_t ds_kmaj = smem_desc(sbase + C::OFF_DS, 16, 1024);
+      const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::PT, 1024);
       // S^T and dP^T of sub-tile u into its stream's columns
-      auto issue_s = [&](int u) -> bool {
+      auto issue_s = [&](int u) {
         const int k = u & 1, stage = u % 3;
-        if (!mbar_wait(&bars->qdo_full[stage], (u / 3) & 1)) return false;
-        if (u >= 2 && !mbar_wait(&bars->tmem_free[k], ((u >> 1) - 1) & 1)) return false;
         tc_fence_after();
         const uint64_t qd = desc_at(q_kmaj, stage * 2 * C::QTILE), dd = desc_at(qd, C::QTILE);
         const uint32_t st = tmem + C::TM_ST + 128 * k;
@@ -628,34 +641,33 @@ __global__ void __launch_bounds__(kThreads, 1)
           tc_mma_ss(st + 64, desc_at(v_kmaj, ko), desc_at(dd, qo), C::IDESC_S, kk > 0);
         }
         tc_commit(&bars->s_full[k]);
-        return true;
       };
-      // dV += P^T dO, dK += dS^T Q, dQ^T = K^T dS^T for sub-tile u
-      auto issue_kv = [&](int u) -> bool {
+      // dQ^T = K^T dS^T (first, so that the drain starts early), then
+      // dV += P^T dO (P^T read from TMEM) and dK += dS^T Q for sub-tile u
+      auto issue_kv = [&](int u) {
         const int k = u & 1, stage = u % 3;
-        if (!mbar_wait(&bars->p_full[k], (u >> 1) & 1)) return false;
         tc_fence_after();
         const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::QTILE), dmn = desc_at(qmn, C::QTILE);
-        const uint64_t pd = desc_at(p_kmaj, 2 * k * C::PT), sd = desc_at(pd, C::PT);
-        const uint64_t smn = desc_at(ds_mnmaj, 2 * k * C::PT);
+        const uint64_t dsk = desc_at(ds_kmaj, k * C::PT), dsm = desc_at(ds_mnmaj, k * C::PT);
+        const uint32_t st = tmem + C::TM_ST + 128 * k;
         const uint32_t acc0 = u > 0 ? 1u : 0u;
 #pragma unroll
-        for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DV, desc_at(pd, kk * 32), desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
-#pragma unroll
-        for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DK, desc_at(sd, kk * 32), desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
-#pragma unroll
         for (int kk = 0; kk < C::BM / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_ST + 128 * k, desc_at(k_mnmaj, kk * 2048), desc_at(smn, kk * 2048), C::IDESC_DQ,
-                    kk > 0 ? 1u : 0u);
+          tc_mma_ss(st, desc_at(k_mnmaj, kk * 2048), desc_at(dsm, kk * 2048), C::IDESC_DQ, kk > 0 ? 1u : 0u);
         tc_commit(&bars->dq_full[k]);
+#pragma unroll
+        for (int kk = 0; kk < C::BQ / 16; ++kk)
+          tc_mma_ts(tmem + C::TM_DV, st + 64 + kk * 8, desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+#pragma unroll
+        for (int kk = 0; kk < C::BQ / 16; ++kk)
+          tc_mma_ss(tmem + C::TM_DK, desc_at(dsk, kk * 32), desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
         tc_commit(&bars->qdo_empty[stage]);
-        return true;
       };
       // issue S(u) and KV(u) in order of u each, whichever is ready first:
       //   S(u) needs Q/dO of u and the stream's TMEM columns back (dQ^T of u-2 drained)
       //   KV(u) needs P^T/dS^T of u
+      // In-order execution of the tensor pipe keeps S(u+2) from overwriting P^T
+      // (dP^T columns) or dS^T of u before KV(u) has read them.
       int next_s = 0, next_kv = 0;
       long long idle_since = clock64();
       while (ok && next_kv < U) {
@@ -664,13 +676,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int u = next_s;
           if (mbar_test(&bars->qdo_full[u % 3], (u / 3) & 1) &&
               (u < 2 || mbar_test(&bars->tmem_free[u & 1], ((u >> 1) - 1) & 1))) {
-            ok = issue_s(u);
+            issue_s(u);
             ++next_s;
             progress = true;
           }
         }
-        if (ok && next_kv < next_s && mbar_test(&bars->p_full[next_kv & 1], (next_kv >> 1) & 1)) {
-          ok = issue_kv(next_kv);
+        if (next_kv < next_s && mbar_test(&bars->p_full[next_kv & 1], (next_kv >> 1) & 1)) {
+          issue_kv(next_kv);
           ++next_kv;
           progress = true;
         }
@@ -683,19 +695,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_commit(&bars->acc_done);
       if (!ok) abort_now();
     }
-  } else if (warp >= 4) {
+  } else if (warp < 12) {
     // ------------------------------------------------------------ compute
+    setmaxnreg_inc<C::REG_COMPUTE>();
     const int k = (warp - 4) >> 2;   // stream
     const int quad = warp & 3;
-    const int r = quad * 32 + lane;  // TMEM lane: key row (P phase) / head dim (dQ phase)
+    const int r = quad * 32 + lane;  // TMEM lane: key row
     const int tw = threadIdx.x - 128 - k * 128;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     const uint32_t st_col = C::TM_ST + 128 * k;
     float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 2 * C::BQ;   // -lse*log2e per query
     float* nds_s = nl2_s + C::BQ;                                                 // -D*scale per query
-    uint8_t* stage_buf = smem + C::OFF_PD + 2 * k * C::PT;           // P^T | dS^T, later dQ^T staging
-    const uint32_t pt_row = smem_u32(stage_buf) + r * 128;
-    const uint32_t ds_row = pt_row + C::PT;
+    const uint32_t ds_row = sbase + C::OFF_DS + k * C::PT + r * 128;
     const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
     auto row_terms = [&](int u, float& nl2, float& nds) {
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
@@ -715,10 +726,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0;; ++i) {
       const int u = 2 * i + k;
       if (u >= U) break;
-      const int h = g * G + u / nsub;
       const int qoff = (u % nsub) * C::BQ;           // query offset from the key tile's first row
-      const int q0 = n * C::BM + qoff;               // first query (in-segment position)
-      if (tw == 0 && i > 0) bulk_wait_read();    // the staging block is read before P^T overwrites it
       if (tw < C::BQ) {
         nl2_s[tw] = next_nl2;
         nds_s[tw] = next_nds;
@@ -736,9 +744,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       reg_fence<64>(sv);
       reg_fence<64>(pv);
       const bool diag = qoff < C::BM;                // this sub-tile overlaps the key tile's rows
+      uint32_t pt[32];                               // P^T row r: bf16 pairs (queries 2j, 2j+1)
 #pragma unroll
       for (int ch = 0; ch < 8; ++ch) {
-        uint32_t wp[4], wd[4];
+        uint32_t wd[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int c = ch * 8 + e * 2;
@@ -755,47 +764,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t t = ffma2(f2pack(__uint_as_float(pv[c]), __uint_as_float(pv[c + 1])), sc2, f2pack(nd.x, nd.y));
           float d0, d1;
           f2unpack(fmul2(pp, t), d0, d1);
-          wp[e] = pack_bf16(p0, p1);
+          pt[ch * 4 + e] = pack_bf16(p0, p1);
           wd[e] = pack_bf16(d0, d1);
         }
-        const uint32_t sw = (uint32_t)((ch ^ (r & 7)) << 4);
-        st_shared_v4(pt_row + sw, wp[0], wp[1], wp[2], wp[3]);
-        st_shared_v4(ds_row + sw, wd[0], wd[1], wd[2], wd[3]);
+        st_shared_v4(ds_row + (uint32_t)((ch ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
       }
+      tmem_st_32x32b_x32(trow + st_col + 64, pt);   // P^T over dP^T (already in registers)
+      tmem_st_wait();
       fence_proxy_async_smem();
       tc_fence_before();
       mbar_arrive(&bars->p_full[k]);
       named_bar_sync(1 + k, 128);                      // everyone is done with this sub-tile's row terms
-      // dQ^T: head dim r on the TMEM lane, the sub-tile's 64 queries on the columns
-      if (!mbar_wait(&bars->dq_full[k], i & 1)) { ok = false; break; }
-      tc_fence_after();
-      uint32_t qv[64];
-      tmem_ld_32x32b_x32(trow + st_col, *reinterpret_cast<uint32_t(*)[32]>(&qv[0]));
-      tmem_ld_32x32b_x32(trow + st_col + 32, *reinterpret_cast<uint32_t(*)[32]>(&qv[32]));
-      tmem_ld_wait();
-      reg_fence<64>(qv);
-      tc_fence_before();
-      mbar_arrive(&bars->tmem_free[k]);
-      // stage dQ^T as a [64 queries][128 dims] fp32 block (query rows past the
-      // segment end are exact zeros) and add it to the accumulator with one TMA op
-      float* stg = reinterpret_cast<float*>(stage_buf);
-#pragma unroll
-      for (int c = 0; c < C::BQ; ++c) stg[c * D + r] = __uint_as_float(qv[c]);
-      fence_proxy_async_smem();
-      named_bar_sync(1 + k, 128);
-      if (tw == 0) {
-        tma_reduce_add_3d(&tm_dq, stg, 0, h, start + q0);
-        bulk_commit();
-      }
       if (aborted_now()) { ok = false; break; }
     }
-    if (tw == 0) bulk_wait_all();
     if (ok && !mbar_wait(&bars->acc_done, 0)) ok = false;
     if (!ok) {
       abort_now();
     } else {
       tc_fence_after();
-      // warpgroup 0 writes dK, warpgroup 1 writes dV (key row r on the TMEM lane)
+      // warpgroup 1 writes dK, warpgroup 2 writes dV (key row r on the TMEM lane)
       const int kpos = n * C::BM + r;
       const uint32_t col = k == 0 ? C::TM_DK : C::TM_DV;
       __nv_bfloat16* outp = (k == 0 ? dk : dv) + ((size_t)(start + kpos) * hkv + g) * D;
@@ -819,6 +806,47 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
+  } else {
+    // ------------------------------------------------------------ dQ drain
+    setmaxnreg_dec<C::REG_DRAIN>();
+    const int dw = threadIdx.x - 12 * 32;
+    float* stg = reinterpret_cast<float*>(smem + C::OFF_STG);
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;  // TMEM lane: head dim
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    bool ok = true;
+    for (int u = 0; u < U; ++u) {
+      const int k = u & 1;
+      const int h = g * G + u / nsub;
+      const int q0 = n * C::BM + (u % nsub) * C::BQ;
+      if (!mbar_wait(&bars->dq_full[k], (u >> 1) & 1)) { ok = false; break; }
+      tc_fence_after();
+      uint32_t a[32], b[32];
+      tmem_ld_32x32b_x32(trow + C::TM_ST + 128 * k, a);
+      tmem_ld_32x32b_x32(trow + C::TM_ST + 128 * k + 32, b);
+      tmem_ld_wait();
+      reg_fence<32>(a);
+      reg_fence<32>(b);
+      tc_fence_before();
+      mbar_arrive(&bars->tmem_free[k]);
+      if (u > 0) {
+        if (dw == 0) bulk_wait_read();
+        named_bar_sync(3, 128);
+      }
+#pragma unroll
+      for (int c = 0; c < 32; ++c) stg[c * D + r] = __uint_as_float(a[c]);
+#pragma unroll
+      for (int c = 0; c < 32; ++c) stg[(32 + c) * D + r] = __uint_as_float(b[c]);
+      fence_proxy_async_smem();
+      named_bar_sync(3, 128);
+      if (dw == 0) {
+        tma_reduce_add_3d(&tm_dq, stg, 0, h, start + q0);
+        bulk_commit();
+      }
+      if (aborted_now()) { ok = false; break; }
+    }
+    if (dw == 0) bulk_wait_all();
+    if (!ok) abort_now();
   }
 
   tc_fence_before();
@@ -860,18 +888,27 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
   if (ntiles > 0) {
     if (D == 128) {
-      alignas(64) CUtensorMap tq64, tdo64, tdq;  // 64-row query sub-tiles; fp32 dQ accumulator
+      alignas(64) CUtensorMap tq64, tdo64, tdq;  // 64-row query sub-tiles
       if (!encode_tma_3d_bf16(&tq64, a.q, D, a.hq, a.num_tokens, 64, 64) ||
           !encode_tma_3d_bf16(&tdo64, dout, D, a.hq, a.num_tokens, 64, 64) ||
           !encode_tma_3d_f32(&tdq, dq_acc, D, a.hq, a.num_tokens, D, 64))
         return cudaErrorInvalidValue;
-      cudaError_t e = cudaFuncSetAttribute(bwd_main_v2, cudaFuncAttributeMaxDynamicSharedMemorySize, V2::SMEM);
+      // the warpgroups' setmaxnreg targets are served from the registers the
+      // block is launched with: refuse to launch a build that got fewer
+      static int regs_ok = -1;
+      if (regs_ok < 0) {
+        cudaFuncAttributes fa;
+        cudaError_t e = cudaFuncGetAttributes(&fa, bwd_main_d128);
+        if (e != cudaSuccess) return e;
+        regs_ok = fa.numRegs == D128::REG_LAUNCH ? 1 : 0;
+      }
+      if (!regs_ok) return cudaErrorInvalidConfiguration;
+      cudaError_t e = cudaFuncSetAttribute(bwd_main_d128, cudaFuncAttributeMaxDynamicSharedMemorySize, D128::SMEM);
       if (e != cudaSuccess) return e;
-      bwd_main_v2<<<grid, kThreads, V2::SMEM, st>>>(tq64, tk, tv, tdo64, tdq, a.cu_seqlens, a.num_segments,
-                                                    (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, a.scale,
-                                                    a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
-                                                    static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
-                                                    a.status);
+      bwd_main_d128<<<grid, D128::THREADS, D128::SMEM, st>>>(
+          tq64, tk, tv, tdo64, tdq, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv,
+          a.scale, a.scale * 1.4426950408889634f, lse, dvec, dq_acc, static_cast<__nv_bfloat16*>(dk),
+          static_cast<__nv_bfloat16*>(dv), a.status);
     } else {
       cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
       if (e != cudaSuccess) return e;
