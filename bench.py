@@ -217,41 +217,46 @@ class Path:
         launches = 0
         for ci in self.chunk_in:
             nseg, ntok = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"]
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)] if ev is not None else None
+            if evs:
+                evs[0].record(tstream)
             st = vcs.vcs_build_segments(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"],
                                         self.window, self.keep, self.max_seg, self.max_tok, self.cu_seqlens, None,
                                         self.tok_gather, self.tok_src, self.tok_pos, self.tok_mask, self.sizes,
                                         self.seg_ws, self.seg_ws_bytes, stream)
             launches += 5
             assert st == 0, vcs.vcs_status_string(st)
+            if evs:
+                evs[1].record(tstream)
             # the attention launch shape depends on the layout sizes: read them (one sync per chunk)
             sz = self.sizes.cpu()
             assert int(sz[0]) == nseg and int(sz[1]) == ntok and (int(sz[2]) >> 32) == 0
             qt = self.q_traj[ci["ttok0"]:ci["ttok1"]]
             kt = self.k_traj[ci["ttok0"]:ci["ttok1"]]
             vt = self.v_traj[ci["ttok0"]:ci["ttok1"]]
+            if evs:
+                evs[2].record(tstream)
             st = vcs.vcs_gather(qt, kt, vt, ci["ttok1"] - ci["ttok0"], self.tok_gather, ntok, hq, hkv, d, self.q,
                                 self.k, self.v, self.gstatus, stream)
             launches += 3
             assert st == 0
-            e0 = e1 = e2 = None
-            if ev is not None:
-                e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
-                e0.record(tstream)
+            if evs:
+                evs[3].record(tstream)
             st = vcs.vcs_attn_fwd(self.q, self.k, self.v, self.cu_seqlens, nseg, ntok, ci["max_seqlen"], hq, hkv,
                                   d, 0.0, self.o, self.lse, self.fwd_ws, self.fwd_ws_bytes, stream)
             launches += 1
             assert st == 0
-            if ev is not None:
-                e1.record(tstream)
+            if evs:
+                evs[4].record(tstream)
             dout = self.dout[ci["tok0"]:ci["tok1"]]
             st = vcs.vcs_attn_bwd(self.q, self.k, self.v, self.o, self.lse, dout, self.cu_seqlens, nseg, ntok,
                                   ci["max_seqlen"], hq, hkv, d, 0.0, self.dq, self.dk, self.dv, self.bwd_ws,
                                   self.bwd_ws_bytes, stream)
             launches += 3
             assert st == 0
-            if ev is not None:
-                e2.record(tstream)
-                ev.append((e0, e1, e2, ci))
+            if evs:
+                evs[5].record(tstream)
+                ev.append((evs, ci))
         self.launches_per_step = launches
 
     def device_status(self):
@@ -374,9 +379,13 @@ def main():
         tt = torch.tensor([ms], device=dev)
         torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
         ms = float(tt.item())
-    fwd_ms = sum(a.elapsed_time(b) for a, b, c, _ in ev) / args.steps
-    bwd_ms = sum(b.elapsed_time(c) for a, b, c, _ in ev) / args.steps
-    bwd_launch_ms = statistics.mean(b.elapsed_time(c) for a, b, c, _ in ev)
+    # per chunk: [0]-[1] build, (host reads the sizes), [2]-[3] gather, [3]-[4] fwd, [4]-[5] bwd
+    build_ms = sum(e[0].elapsed_time(e[1]) for e, _ in ev) / args.steps
+    gather_ms = sum(e[2].elapsed_time(e[3]) for e, _ in ev) / args.steps
+    fwd_ms = sum(e[3].elapsed_time(e[4]) for e, _ in ev) / args.steps
+    bwd_ms = sum(e[4].elapsed_time(e[5]) for e, _ in ev) / args.steps
+    bwd_launch_ms = statistics.mean(e[4].elapsed_time(e[5]) for e, _ in ev)
+    gather_bytes = path.num_tokens * 2 * (w.hq + 2 * w.hkv) * w.d * 2     # rows read once + written once
     bwd_launch_flops = f_bwd / len(path.chunk_in)
 
     value = flops * world / (ms / 1e3) / 1e12
@@ -398,6 +407,7 @@ def main():
                    "max_seqlen": int(path.seg_lens.max()), "chunks": len(path.chunk_in),
                    "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)"},
         "attn_tflop_credited": flops / 1e12,
+        "builder_ms": build_ms, "gather_ms": gather_ms, "gather_gbs": gather_bytes / (gather_ms / 1e3) / 1e9,
         "attn_fwd_ms": fwd_ms, "attn_bwd_ms": bwd_ms,
         "attn_fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "attn_bwd_tflops": f_bwd / (bwd_ms / 1e3) / 1e12,
         "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,

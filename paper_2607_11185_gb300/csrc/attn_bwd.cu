@@ -483,8 +483,8 @@ static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D1
 
 struct D128Bars {
   uint64_t kv_full;
-  uint64_t qdo_full[3];
-  uint64_t qdo_empty[3];
+  uint64_t qdo_full[D128::NST];
+  uint64_t qdo_empty[D128::NST];
   uint64_t s_full[2];
   uint64_t p_full[2];
   uint64_t dq_full[2];
@@ -545,13 +545,21 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   const int G = hq / hkv;
   const int nsub = (L - n * C::BM + C::BQ - 1) / C::BQ;  // 64-row query sub-tiles at or after this key tile
   const int U = G * nsub;
+  // Sub-tile u covers query rows n*BM + sub_of(u)*BQ ... +BQ-1 of head head_of(u).
+  // Rows are swept from the segment end toward the key tile, the G heads of
+  // one row block in turn: the CTAs of one (segment, kv head) that run at the
+  // same time then work on the same query rows together, so their Q/dO loads
+  // and dQ reduce-adds meet the same L2 lines instead of each CTA streaming
+  // its own part of the accumulator through HBM.
+  auto sub_of = [&](int u) { return nsub - 1 - u / G; };
+  auto head_of = [&](int u) { return g * G + u % G; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t sbase = smem_u32(smem);
 
   if (threadIdx.x == 0) {
     mbar_init(&bars->kv_full, 1);
-    for (int i = 0; i < 3; ++i) {
+    for (int i = 0; i < C::NST; ++i) {
       mbar_init(&bars->qdo_full[i], 1);
       mbar_init(&bars->qdo_empty[i], 1);
     }
@@ -594,10 +602,10 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         tma_load_3d(smem + C::OFF_V + kb * C::KVBLOCK, &tm_v, &bars->kv_full, kb * 64, g, start + n * C::BM);
       }
       for (int u = 0; u < U; ++u) {
-        const int h = g * G + u / nsub;
-        const int q0 = n * C::BM + (u % nsub) * C::BQ;
-        const int stage = u % 3;
-        if (u >= 3 && !mbar_wait(&bars->qdo_empty[stage], ((u / 3) - 1) & 1)) {
+        const int h = head_of(u);
+        const int q0 = n * C::BM + sub_of(u) * C::BQ;
+        const int stage = u % C::NST;
+        if (u >= C::NST && !mbar_wait(&bars->qdo_empty[stage], ((u / C::NST) - 1) & 1)) {
           abort_now();
           break;
         }
@@ -624,7 +632,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::PT, 1024);
       // S^T and dP^T of sub-tile u into its stream's columns
       auto issue_s = [&](int u) {
-        const int k = u & 1, stage = u % 3;
+        const int k = u & 1, stage = u % C::NST;
         tc_fence_after();
         const uint64_t qd = desc_at(q_kmaj, stage * 2 * C::QTILE), dd = desc_at(qd, C::QTILE);
         const uint32_t st = tmem + C::TM_ST + 128 * k;
@@ -645,7 +653,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       // dQ^T = K^T dS^T (first, so that the drain starts early), then
       // dV += P^T dO (P^T read from TMEM) and dK += dS^T Q for sub-tile u
       auto issue_kv = [&](int u) {
-        const int k = u & 1, stage = u % 3;
+        const int k = u & 1, stage = u % C::NST;
         tc_fence_after();
         const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::QTILE), dmn = desc_at(qmn, C::QTILE);
         const uint64_t dsk = desc_at(ds_kmaj, k * C::PT), dsm = desc_at(ds_mnmaj, k * C::PT);
@@ -674,7 +682,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         bool progress = false;
         if (next_s < U && next_s <= next_kv + 1) {
           const int u = next_s;
-          if (mbar_test(&bars->qdo_full[u % 3], (u / 3) & 1) &&
+          if (mbar_test(&bars->qdo_full[u % C::NST], (u / C::NST) & 1) &&
               (u < 2 || mbar_test(&bars->tmem_free[u & 1], ((u >> 1) - 1) & 1))) {
             issue_s(u);
             ++next_s;
@@ -712,8 +720,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
       nds = 0.f;
       if (u < U && tw < C::BQ) {
-        const int h = g * G + u / nsub;
-        const int q = n * C::BM + (u % nsub) * C::BQ + tw;
+        const int h = head_of(u);
+        const int q = n * C::BM + sub_of(u) * C::BQ + tw;
         if (q < L) {
           nl2 = -__ldg(&lse[(size_t)h * num_tokens + start + q]) * 1.4426950408889634f;
           nds = -__ldg(&dvec[(size_t)h * num_tokens + start + q]) * scale;
@@ -726,7 +734,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     for (int i = 0;; ++i) {
       const int u = 2 * i + k;
       if (u >= U) break;
-      const int qoff = (u % nsub) * C::BQ;           // query offset from the key tile's first row
+      const int qoff = sub_of(u) * C::BQ;            // query offset from the key tile's first row
       if (tw < C::BQ) {
         nl2_s[tw] = next_nl2;
         nds_s[tw] = next_nds;
@@ -817,8 +825,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     bool ok = true;
     for (int u = 0; u < U; ++u) {
       const int k = u & 1;
-      const int h = g * G + u / nsub;
-      const int q0 = n * C::BM + (u % nsub) * C::BQ;
+      const int h = head_of(u);
+      const int q0 = n * C::BM + sub_of(u) * C::BQ;
       if (!mbar_wait(&bars->dq_full[k], (u >> 1) & 1)) { ok = false; break; }
       tc_fence_after();
       uint32_t a[32], b[32];
