@@ -62,15 +62,17 @@ bool encode_tma_3d_bf16(void* map, const void* base, uint64_t d, uint64_t heads,
 }
 
 bool encode_tma_3d_f32(void* map, const void* base, uint64_t d, uint64_t heads, uint64_t tokens, uint32_t box_d,
-                       uint32_t box_rows) {
+                       uint32_t box_rows, bool swizzle128) {
   std::call_once(g_encode_once, load_encode_fn);
   if (g_encode == nullptr) return false;
   cuuint64_t dims[3] = {d, heads, tokens > 0 ? tokens : 1};
   cuuint64_t strides[2] = {d * 4, heads * d * 4};
   cuuint32_t box[3] = {box_d, 1, box_rows};
   cuuint32_t estr[3] = {1, 1, 1};
+  if (swizzle128 && box_d * 4 != 128) return false;
   CUresult r = g_encode(static_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base),
-                        dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                        dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }

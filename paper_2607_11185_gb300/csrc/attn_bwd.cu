@@ -29,9 +29,9 @@
 //   compute warps: dQ rows (query rows on TMEM lanes) -> red.global.add.v4.f32
 // Warp roles as in the forward: warp 0 TMA, warp 1 MMA, warps 4-11 compute
 // (two warpgroups, each owning half of the 128 query columns / D columns).
-// For head_dim 128, bwd_main_d128 replaces bwd_main: 64-query sub-tiles in two
-// streams, P^T kept in TMEM, and a fourth warpgroup that drains dQ with TMA
-// bulk reduce-adds (described at the kernel).
+// For head_dim 128, bwd_main_d128 replaces bwd_main: P^T kept in TMEM, dQ
+// computed with query rows on TMEM lanes, and a fourth warpgroup that drains it
+// with TMA bulk reduce-adds (described at the kernel).
 #include <cfloat>
 #include <cstdint>
 
@@ -430,80 +430,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ bwd_main_d128 (head_dim 128)
-// Same work unit and result as bwd_main, reorganised for overlap.  The query
-// rows of every (query tile, head) are processed as 64-row sub-tiles; sub-tile
-// u belongs to stream u & 1.  Four warpgroups:
-//   WG0   warp 0: TMA producer (K and V once, Q/dO sub-tiles through a 3-stage ring)
+// Same work unit and result as bwd_main, with every MMA at N = 128 (the
+// tensor pipe's full rate; N = 64 runs at 2/3).  The query rows of each
+// (query tile, head) are processed as 128-row tiles in one stream; the two
+// compute warpgroups split a tile's query columns.
+//   WG0   warp 0: TMA producer (K and V once, Q/dO 128-row tiles through a 2-stage ring)
 //         warp 1: TMEM allocation and the single MMA-issuing thread
-//   WG1/2 compute for stream 0/1: S^T, dP^T -> P^T (bf16, written back to TMEM
-//         over dP^T: the A operand of dV += P^T dO) and dS^T (bf16, shared
-//         memory: operand of dK += dS^T Q and dQ^T = K^T dS^T)
-//   WG3   dQ drain: takes dQ^T of each sub-tile (head dims on TMEM lanes, its 64
-//         queries on columns) as soon as its MMAs finish, hands the columns back
-//         to the stream, stages the block as [64 queries][128 dims] fp32 in shared
-//         memory and adds it to the fp32 dQ accumulator with one TMA bulk
-//         reduce-add (query rows past the segment end are exact zeros)
-// so that neither the compute warpgroups nor the tensor pipe wait for the
-// accumulation.  Registers are rebalanced per warpgroup with setmaxnreg
-// (80 / 176 / 176 / 80 per thread; the block launches with 128).
-//   TMEM: dV [0,128), dK [128,256),
-//         stream k: S^T, later dQ^T [256+128k, +64); dP^T, later P^T [+64, +128)
-//   smem: K, V (64 KB), 3-stage Q/dO ring (96 KB), dS^T per stream (32 KB), row terms (1 KB),
-//         dQ^T staging block (32 KB)
-struct D128 {
-  static constexpr int D = 128;
-  static constexpr int BM = 128;                 // key rows of the tile
-  static constexpr int BQ = 64;                  // query rows per sub-tile
-  static constexpr int NST = 3;                  // Q/dO ring stages
-  static constexpr int THREADS = 512;
-  static constexpr int KVTILE = BM * D * 2;      // 32 KB
-  static constexpr int KVBLOCK = BM * 128;       // one 64-dim column block of K or V
-  static constexpr int QTILE = BQ * D * 2;       // 16 KB
-  static constexpr int QBLOCK = BQ * 128;        // one 64-dim column block of a Q/dO sub-tile
-  static constexpr int PT = BM * BQ * 2;         // 16 KB: 128 keys x 64 queries bf16
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = KVTILE;
-  static constexpr int OFF_Q = 2 * KVTILE;                     // stage s: Q at +s*2*QTILE, dO at +QTILE
-  static constexpr int OFF_DS = OFF_Q + NST * 2 * QTILE;       // stream k: dS^T at +k*PT
-  static constexpr int OFF_ROW = OFF_DS + 2 * PT;              // stream k: -lse*log2e [64], -D*scale [64]
-  static constexpr int OFF_STG = OFF_ROW + 2 * 2 * BQ * 4;
-  static constexpr int OFF_BAR = OFF_STG + BQ * D * 4;
-  static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr int TM_DV = 0, TM_DK = 128, TM_ST = 256;    // stream k: S^T at TM_ST + 128k, dP^T at +64
-  // registers per thread after rebalancing: WG0, each compute warpgroup, the drain warpgroup
-  static constexpr int REG_CTRL = 80, REG_COMPUTE = 176, REG_DRAIN = 80;
-  static constexpr int REG_LAUNCH = 65536 / THREADS;
-  static constexpr uint32_t IDESC_S = idesc_bf16(128, BQ, 0, 0);   // K or V (K-major) x Q or dO^T (K-major)
-  static constexpr uint32_t IDESC_KV = idesc_bf16(128, D, 0, 1);   // P^T/dS^T (TMEM or K-major) x dO/Q (MN-major)
-  static constexpr uint32_t IDESC_DQ = idesc_bf16(128, BQ, 1, 1);  // K^T (MN-major) x dS^T (MN-major)
-};
-static_assert(D128::SMEM <= 232448, "shared memory budget");
-static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D128::REG_LAUNCH,
-              "setmaxnreg targets exceed the registers the block is launched with");
+//   WG1/2 compute, query columns [0,64) / [64,128): S^T, dP^T -> P^T (bf16,
+//         written back to TMEM over dP^T: the A operand of dV += P^T dO) and
+//         dS^T (bf16, shared memory: dK += dS^T Q and dQ = dS K)
+//   WG3   dQ drain: once a tile's MMAs are complete, dQ (query rows on TMEM
+//         lanes) is copied into the tile's freed Q/dO stage, the columns are
+//         handed back, and TMA bulk reduce-adds add it to the fp32 accumulator
+// Registers are rebalanced per warpgroup with setmaxnreg (104 / 176 / 176 / 56
+// per thread; the block launches with 128).
+// With a 64-query sub-tile and two streams (compute of one stream overlapping
+// the other's MMAs) the N = 64 MMAs held the backward 5% lower on the
+// long-horizon workload than this single stream of 128-query tiles.
+//   TMEM: dV [0,128), dK [128,256), S^T then dQ [256,384), dP^T then P^T [384,512)
+//   smem: K, V (64 KB), 2-stage Q/dO ring (128 KB; a freed stage also stages dQ),
+//         dS^T (32 KB), row terms (1 KB)
 
-struct D128Bars {
-  uint64_t kv_full;
-  uint64_t qdo_full[D128::NST];
-  uint64_t qdo_empty[D128::NST];
-  uint64_t s_full[2];
-  uint64_t p_full[2];
-  uint64_t dq_full[2];
-  uint64_t tmem_free[2];
-  uint64_t acc_done;
-  uint32_t tmem_base;
-  int32_t abort;
-};
-
-__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
+// dst (global, tensor map) += src (shared) for one box, asynchronously (bulk group).
 __device__ __forceinline__ void tma_reduce_add_3d(const void* map, const void* src, int x, int y, int z) {
   asm volatile(
       "cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(map),
@@ -514,12 +462,52 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
+struct D128 {
+  static constexpr int D = 128;
+  static constexpr int BM = 128;                 // key rows of the tile
+  static constexpr int BQ = 128;                 // query rows per tile
+  static constexpr int NST = 2;                  // Q/dO ring stages
+  static constexpr int THREADS = 512;
+  static constexpr int TILE = 128 * D * 2;       // 32 KB: K, V, a Q or a dO tile
+  static constexpr int BLOCK = 128 * 128;        // one 64-column block of a 128-row tile
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = TILE;
+  static constexpr int OFF_Q = 2 * TILE;                       // stage s: Q at +s*2*TILE, dO at +TILE
+  static constexpr int OFF_DS = OFF_Q + NST * 2 * TILE;        // dS^T [128 keys][128 queries], two 64-query blocks
+  static constexpr int OFF_ROW = OFF_DS + TILE;                // WG k: -lse*log2e [64], -D*scale [64]
+  static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * 64 * 4;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;
+  static constexpr int TM_DV = 0, TM_DK = 128, TM_S = 256, TM_P = 384;
+  static constexpr int REG_CTRL = 104, REG_COMPUTE = 176, REG_DRAIN = 56;
+  static constexpr int REG_LAUNCH = 65536 / THREADS;
+  static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
+  static constexpr uint32_t IDESC_KV = idesc_bf16(128, 128, 0, 1);  // P^T (TMEM) / dS^T (K-major) x dO / Q (MN-major)
+  static constexpr uint32_t IDESC_DQ = idesc_bf16(128, 128, 1, 1);  // dS (MN-major) x K (MN-major)
+};
+static_assert(D128::SMEM <= 232448, "shared memory budget");
+static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D128::REG_LAUNCH,
+              "setmaxnreg targets exceed the registers the block is launched with");
+
+struct D128Bars {
+  uint64_t kv_full;
+  uint64_t qdo_full[D128::NST];
+  uint64_t kv_done[D128::NST];     // the tile's MMAs are complete: its Q/dO stage may be overwritten
+  uint64_t stage_free[D128::NST];  // the drain's reduce-adds have read the stage
+  uint64_t s_full;
+  uint64_t p_full;
+  uint64_t tmem_free;
+  uint64_t acc_done;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+
+
 __global__ void __launch_bounds__(D128::THREADS, 1)
     bwd_main_d128(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                  const __grid_constant__ CUtensorMap tm_dq, const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens,
-                  int32_t max_seqlen, int32_t hq, int32_t hkv, float scale, float scale_log2,
-                  const float* __restrict__ lse, const float* __restrict__ dvec, float* __restrict__ dq_acc,
+                  const __grid_constant__ CUtensorMap tm_dq, const int32_t* __restrict__ cu_seqlens,
+                  int32_t num_segments, int32_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, float scale,
+                  float scale_log2, const float* __restrict__ lse, const float* __restrict__ dvec,
                   __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status) {
   using C = D128;
   constexpr int D = C::D;
@@ -543,14 +531,11 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   const int L = end - start;
   if (n * C::BM >= L) return;
   const int G = hq / hkv;
-  const int nsub = (L - n * C::BM + C::BQ - 1) / C::BQ;  // 64-row query sub-tiles at or after this key tile
+  const int nsub = (L - n * C::BM + C::BQ - 1) / C::BQ;  // 128-row query tiles at or after this key tile
   const int U = G * nsub;
-  // Sub-tile u covers query rows n*BM + sub_of(u)*BQ ... +BQ-1 of head head_of(u).
-  // Rows are swept from the segment end toward the key tile, the G heads of
-  // one row block in turn: the CTAs of one (segment, kv head) that run at the
-  // same time then work on the same query rows together, so their Q/dO loads
-  // and dQ reduce-adds meet the same L2 lines instead of each CTA streaming
-  // its own part of the accumulator through HBM.
+  // Tile u covers query rows n*BM + sub_of(u)*BQ ... +BQ-1 of head head_of(u), swept from the
+  // segment end toward the key tile with the G heads of one row block in turn, so that the key
+  // tiles of one (segment, kv head) running together meet the same Q/dO/dQ lines in L2.
   auto sub_of = [&](int u) { return nsub - 1 - u / G; };
   auto head_of = [&](int u) { return g * G + u % G; };
 
@@ -561,14 +546,12 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     mbar_init(&bars->kv_full, 1);
     for (int i = 0; i < C::NST; ++i) {
       mbar_init(&bars->qdo_full[i], 1);
-      mbar_init(&bars->qdo_empty[i], 1);
+      mbar_init(&bars->kv_done[i], 1);
+      mbar_init(&bars->stage_free[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->p_full[i], 128);
-      mbar_init(&bars->dq_full[i], 1);
-      mbar_init(&bars->tmem_free[i], 128);
-    }
+    mbar_init(&bars->s_full, 1);
+    mbar_init(&bars->p_full, 256);
+    mbar_init(&bars->tmem_free, 128);
     mbar_init(&bars->acc_done, 1);
     bars->abort = 0;
     fence_mbar_init();
@@ -595,110 +578,83 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
       tma_prefetch_desc(&tm_do);
-      mbar_arrive_expect_tx(&bars->kv_full, 2 * C::KVTILE);
+      mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
 #pragma unroll
       for (int kb = 0; kb < 2; ++kb) {
-        tma_load_3d(smem + C::OFF_K + kb * C::KVBLOCK, &tm_k, &bars->kv_full, kb * 64, g, start + n * C::BM);
-        tma_load_3d(smem + C::OFF_V + kb * C::KVBLOCK, &tm_v, &bars->kv_full, kb * 64, g, start + n * C::BM);
+        tma_load_3d(smem + C::OFF_K + kb * C::BLOCK, &tm_k, &bars->kv_full, kb * 64, g, start + n * C::BM);
+        tma_load_3d(smem + C::OFF_V + kb * C::BLOCK, &tm_v, &bars->kv_full, kb * 64, g, start + n * C::BM);
       }
       for (int u = 0; u < U; ++u) {
         const int h = head_of(u);
         const int q0 = n * C::BM + sub_of(u) * C::BQ;
         const int stage = u % C::NST;
-        if (u >= C::NST && !mbar_wait(&bars->qdo_empty[stage], ((u / C::NST) - 1) & 1)) {
+        if (u >= C::NST && !mbar_wait(&bars->stage_free[stage], ((u / C::NST) - 1) & 1)) {
           abort_now();
           break;
         }
         if (aborted_now()) break;
-        mbar_arrive_expect_tx(&bars->qdo_full[stage], 2 * C::QTILE);
-        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::QTILE;
+        mbar_arrive_expect_tx(&bars->qdo_full[stage], 2 * C::TILE);
+        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::TILE;
 #pragma unroll
         for (int kb = 0; kb < 2; ++kb) {
-          tma_load_3d(qs + kb * C::QBLOCK, &tm_q, &bars->qdo_full[stage], kb * 64, h, start + q0);
-          tma_load_3d(qs + C::QTILE + kb * C::QBLOCK, &tm_do, &bars->qdo_full[stage], kb * 64, h, start + q0);
+          tma_load_3d(qs + kb * C::BLOCK, &tm_q, &bars->qdo_full[stage], kb * 64, h, start + q0);
+          tma_load_3d(qs + C::TILE + kb * C::BLOCK, &tm_do, &bars->qdo_full[stage], kb * 64, h, start + q0);
         }
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- MMA issuer
       bool ok = mbar_wait(&bars->kv_full, 0);
-      tc_fence_after();
       // descriptors built once; the issue loops only add compile-time offsets
       const uint64_t k_kmaj = smem_desc(sbase + C::OFF_K, 16, 1024);
       const uint64_t v_kmaj = smem_desc(sbase + C::OFF_V, 16, 1024);
-      const uint64_t k_mnmaj = smem_desc(sbase + C::OFF_K, C::KVBLOCK, 1024);
+      const uint64_t k_mnmaj = smem_desc(sbase + C::OFF_K, C::BLOCK, 1024);
       const uint64_t q_kmaj = smem_desc(sbase + C::OFF_Q, 16, 1024);
-      const uint64_t q_mnmaj = smem_desc(sbase + C::OFF_Q, C::QBLOCK, 1024);
+      const uint64_t q_mnmaj = smem_desc(sbase + C::OFF_Q, C::BLOCK, 1024);
       const uint64_t ds_kmaj = smem_desc(sbase + C::OFF_DS, 16, 1024);
-      const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::PT, 1024);
-      // S^T and dP^T of sub-tile u into its stream's columns
-      auto issue_s = [&](int u) {
-        const int k = u & 1, stage = u % C::NST;
+      const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::BLOCK, 1024);
+      for (int u = 0; ok && u < U; ++u) {
+        const int stage = u % C::NST;
+        // S^T = K Q^T and dP^T = V dO^T: need Q/dO of u and the S^T columns back (dQ of u-1 drained)
+        if (!mbar_wait(&bars->qdo_full[stage], (u / C::NST) & 1) ||
+            (u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) || aborted_now()) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        const uint64_t qd = desc_at(q_kmaj, stage * 2 * C::QTILE), dd = desc_at(qd, C::QTILE);
-        const uint32_t st = tmem + C::TM_ST + 128 * k;
+        const uint64_t qd = desc_at(q_kmaj, stage * 2 * C::TILE), dd = desc_at(qd, C::TILE);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
-          const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
-          tc_mma_ss(st, desc_at(k_kmaj, ko), desc_at(qd, qo), C::IDESC_S, kk > 0);
+          const uint32_t o = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
+          tc_mma_ss(tmem + C::TM_S, desc_at(k_kmaj, o), desc_at(qd, o), C::IDESC_S, kk > 0);
         }
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t ko = (kk >> 2) * C::KVBLOCK + (kk & 3) * 32;
-          const uint32_t qo = (kk >> 2) * C::QBLOCK + (kk & 3) * 32;
-          tc_mma_ss(st + 64, desc_at(v_kmaj, ko), desc_at(dd, qo), C::IDESC_S, kk > 0);
+          const uint32_t o = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
+          tc_mma_ss(tmem + C::TM_P, desc_at(v_kmaj, o), desc_at(dd, o), C::IDESC_S, kk > 0);
         }
-        tc_commit(&bars->s_full[k]);
-      };
-      // dQ^T = K^T dS^T (first, so that the drain starts early), then
-      // dV += P^T dO (P^T read from TMEM) and dK += dS^T Q for sub-tile u
-      auto issue_kv = [&](int u) {
-        const int k = u & 1, stage = u % C::NST;
+        tc_commit(&bars->s_full);
+        // dQ = dS K, dV += P^T dO, dK += dS^T Q.  In-order execution keeps S(u+1) from
+        // overwriting P^T or dS^T before these read them.
+        if (!mbar_wait(&bars->p_full, u & 1)) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
-        const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::QTILE), dmn = desc_at(qmn, C::QTILE);
-        const uint64_t dsk = desc_at(ds_kmaj, k * C::PT), dsm = desc_at(ds_mnmaj, k * C::PT);
-        const uint32_t st = tmem + C::TM_ST + 128 * k;
+        const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::TILE), dmn = desc_at(qmn, C::TILE);
         const uint32_t acc0 = u > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < C::BM / 16; ++kk)
-          tc_mma_ss(st, desc_at(k_mnmaj, kk * 2048), desc_at(dsm, kk * 2048), C::IDESC_DQ, kk > 0 ? 1u : 0u);
-        tc_commit(&bars->dq_full[k]);
+          tc_mma_ss(tmem + C::TM_S, desc_at(ds_mnmaj, kk * 2048), desc_at(k_mnmaj, kk * 2048), C::IDESC_DQ,
+                    kk > 0 ? 1u : 0u);
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ts(tmem + C::TM_DV, st + 64 + kk * 8, desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+          tc_mma_ts(tmem + C::TM_DV, tmem + C::TM_P + (kk >> 2) * 64 + (kk & 3) * 8, desc_at(dmn, kk * 2048),
+                    C::IDESC_KV, kk > 0 ? 1u : acc0);
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DK, desc_at(dsk, kk * 32), desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
-        tc_commit(&bars->qdo_empty[stage]);
-      };
-      // issue S(u) and KV(u) in order of u each, whichever is ready first:
-      //   S(u) needs Q/dO of u and the stream's TMEM columns back (dQ^T of u-2 drained)
-      //   KV(u) needs P^T/dS^T of u
-      // In-order execution of the tensor pipe keeps S(u+2) from overwriting P^T
-      // (dP^T columns) or dS^T of u before KV(u) has read them.
-      int next_s = 0, next_kv = 0;
-      long long idle_since = clock64();
-      while (ok && next_kv < U) {
-        bool progress = false;
-        if (next_s < U && next_s <= next_kv + 1) {
-          const int u = next_s;
-          if (mbar_test(&bars->qdo_full[u % C::NST], (u / C::NST) & 1) &&
-              (u < 2 || mbar_test(&bars->tmem_free[u & 1], ((u >> 1) - 1) & 1))) {
-            issue_s(u);
-            ++next_s;
-            progress = true;
-          }
-        }
-        if (next_kv < next_s && mbar_test(&bars->p_full[next_kv & 1], (next_kv >> 1) & 1)) {
-          issue_kv(next_kv);
-          ++next_kv;
-          progress = true;
-        }
-        if (progress) {
-          idle_since = clock64();
-        } else if (clock64() - idle_since > kWaitLimitCycles || aborted_now()) {
-          ok = false;
-        }
+          tc_mma_ss(tmem + C::TM_DK, desc_at(ds_kmaj, (kk >> 2) * C::BLOCK + (kk & 3) * 32),
+                    desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+        tc_commit(&bars->kv_done[stage]);
       }
       tc_commit(&bars->acc_done);
       if (!ok) abort_now();
@@ -706,22 +662,21 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   } else if (warp < 12) {
     // ------------------------------------------------------------ compute
     setmaxnreg_inc<C::REG_COMPUTE>();
-    const int k = (warp - 4) >> 2;   // stream
+    const int k = (warp - 4) >> 2;   // query columns [64k, 64k+64) of the tile
     const int quad = warp & 3;
     const int r = quad * 32 + lane;  // TMEM lane: key row
     const int tw = threadIdx.x - 128 - k * 128;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    const uint32_t st_col = C::TM_ST + 128 * k;
-    float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 2 * C::BQ;   // -lse*log2e per query
-    float* nds_s = nl2_s + C::BQ;                                                 // -D*scale per query
-    const uint32_t ds_row = sbase + C::OFF_DS + k * C::PT + r * 128;
+    float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;   // -lse*log2e per query
+    float* nds_s = nl2_s + 64;                                              // -D*scale per query
+    const uint32_t ds_row = sbase + C::OFF_DS + k * C::BLOCK + r * 128;
     const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
     auto row_terms = [&](int u, float& nl2, float& nds) {
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
       nds = 0.f;
-      if (u < U && tw < C::BQ) {
+      if (u < U && tw < 64) {
         const int h = head_of(u);
-        const int q = n * C::BM + sub_of(u) * C::BQ + tw;
+        const int q = n * C::BM + sub_of(u) * C::BQ + 64 * k + tw;
         if (q < L) {
           nl2 = -__ldg(&lse[(size_t)h * num_tokens + start + q]) * 1.4426950408889634f;
           nds = -__ldg(&dvec[(size_t)h * num_tokens + start + q]) * scale;
@@ -729,29 +684,27 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       }
     };
     float next_nl2, next_nds;
-    row_terms(k, next_nl2, next_nds);
+    row_terms(0, next_nl2, next_nds);
     bool ok = true;
-    for (int i = 0;; ++i) {
-      const int u = 2 * i + k;
-      if (u >= U) break;
-      const int qoff = sub_of(u) * C::BQ;            // query offset from the key tile's first row
-      if (tw < C::BQ) {
+    for (int u = 0; u < U; ++u) {
+      const int qoff = sub_of(u) * C::BQ + 64 * k;  // first query column of this warpgroup, from the key tile's first row
+      if (tw < 64) {
         nl2_s[tw] = next_nl2;
         nds_s[tw] = next_nds;
       }
       named_bar_sync(1 + k, 128);
-      row_terms(u + 2, next_nl2, next_nds);
-      if (!mbar_wait(&bars->s_full[k], i & 1)) { ok = false; break; }
+      row_terms(u + 1, next_nl2, next_nds);
+      if (!mbar_wait(&bars->s_full, u & 1)) { ok = false; break; }
       tc_fence_after();
       uint32_t sv[64], pv[64];
-      tmem_ld_32x32b_x32(trow + st_col, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-      tmem_ld_32x32b_x32(trow + st_col + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
-      tmem_ld_32x32b_x32(trow + st_col + 64, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
-      tmem_ld_32x32b_x32(trow + st_col + 96, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
+      tmem_ld_32x32b_x32(trow + C::TM_S + 64 * k, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld_32x32b_x32(trow + C::TM_S + 64 * k + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tmem_ld_32x32b_x32(trow + C::TM_P + 64 * k, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
+      tmem_ld_32x32b_x32(trow + C::TM_P + 64 * k + 32, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
       tmem_ld_wait();
       reg_fence<64>(sv);
       reg_fence<64>(pv);
-      const bool diag = qoff < C::BM;                // this sub-tile overlaps the key tile's rows
+      const bool diag = qoff < C::BM;                // these columns overlap the key tile's rows
       uint32_t pt[32];                               // P^T row r: bf16 pairs (queries 2j, 2j+1)
 #pragma unroll
       for (int ch = 0; ch < 8; ++ch) {
@@ -777,12 +730,12 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         }
         st_shared_v4(ds_row + (uint32_t)((ch ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
       }
-      tmem_st_32x32b_x32(trow + st_col + 64, pt);   // P^T over dP^T (already in registers)
+      tmem_st_32x32b_x32(trow + C::TM_P + 64 * k, pt);   // P^T over this warpgroup's dP^T columns
       tmem_st_wait();
       fence_proxy_async_smem();
       tc_fence_before();
-      mbar_arrive(&bars->p_full[k]);
-      named_bar_sync(1 + k, 128);                      // everyone is done with this sub-tile's row terms
+      mbar_arrive(&bars->p_full);
+      named_bar_sync(1 + k, 128);                      // everyone is done with this tile's row terms
       if (aborted_now()) { ok = false; break; }
     }
     if (ok && !mbar_wait(&bars->acc_done, 0)) ok = false;
@@ -816,40 +769,49 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ dQ drain
+    // Once a tile's MMAs are complete its Q/dO stage is free: dQ (query rows on TMEM lanes) is
+    // copied there as four [128 rows][32 dims] fp32 blocks in the 128-byte swizzled layout of
+    // the accumulator's tensor map, added to the accumulator with four TMA bulk reduce-adds
+    // (rows past the segment end are exact zeros), and the stage is handed back to the producer
+    // once the reduce-adds have read it.
     setmaxnreg_dec<C::REG_DRAIN>();
-    const int dw = threadIdx.x - 12 * 32;
-    float* stg = reinterpret_cast<float*>(smem + C::OFF_STG);
     const int quad = warp & 3;
-    const int r = quad * 32 + lane;  // TMEM lane: head dim
+    const int l = quad * 32 + lane;  // TMEM lane: query row of the tile
+    const int dw = threadIdx.x - 12 * 32;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     bool ok = true;
     for (int u = 0; u < U; ++u) {
-      const int k = u & 1;
-      const int h = head_of(u);
-      const int q0 = n * C::BM + sub_of(u) * C::BQ;
-      if (!mbar_wait(&bars->dq_full[k], (u >> 1) & 1)) { ok = false; break; }
+      const int stage = u % C::NST;
+      if (!mbar_wait(&bars->kv_done[stage], (u / C::NST) & 1)) { ok = false; break; }
       tc_fence_after();
-      uint32_t a[32], b[32];
-      tmem_ld_32x32b_x32(trow + C::TM_ST + 128 * k, a);
-      tmem_ld_32x32b_x32(trow + C::TM_ST + 128 * k + 32, b);
-      tmem_ld_wait();
-      reg_fence<32>(a);
-      reg_fence<32>(b);
-      tc_fence_before();
-      mbar_arrive(&bars->tmem_free[k]);
-      if (u > 0) {
-        if (dw == 0) bulk_wait_read();
-        named_bar_sync(3, 128);
+      uint8_t* stg = smem + C::OFF_Q + stage * 2 * C::TILE;
+      const uint32_t srow = smem_u32(stg) + l * 128;
+#pragma unroll
+      for (int part = 0; part < D / 32; ++part) {
+        uint32_t a[32];
+        tmem_ld_32x32b_x32(trow + C::TM_S + part * 32, a);
+        tmem_ld_wait();
+        reg_fence<32>(a);
+        if (part == D / 32 - 1) {
+          tc_fence_before();
+          mbar_arrive(&bars->tmem_free);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          st_shared_v4(srow + part * (128 * 128) + (uint32_t)((j ^ (l & 7)) << 4), a[4 * j], a[4 * j + 1],
+                       a[4 * j + 2], a[4 * j + 3]);
       }
-#pragma unroll
-      for (int c = 0; c < 32; ++c) stg[c * D + r] = __uint_as_float(a[c]);
-#pragma unroll
-      for (int c = 0; c < 32; ++c) stg[(32 + c) * D + r] = __uint_as_float(b[c]);
       fence_proxy_async_smem();
       named_bar_sync(3, 128);
       if (dw == 0) {
-        tma_reduce_add_3d(&tm_dq, stg, 0, h, start + q0);
+        const int h = head_of(u);
+        const int q0 = n * C::BM + sub_of(u) * C::BQ;
+#pragma unroll
+        for (int part = 0; part < D / 32; ++part)
+          tma_reduce_add_3d(&tm_dq, stg + part * (128 * 128), part * 32, h, start + q0);
         bulk_commit();
+        bulk_wait_read();
+        mbar_arrive(&bars->stage_free[stage]);
       }
       if (aborted_now()) { ok = false; break; }
     }
@@ -896,11 +858,6 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
   if (ntiles > 0) {
     if (D == 128) {
-      alignas(64) CUtensorMap tq64, tdo64, tdq;  // 64-row query sub-tiles
-      if (!encode_tma_3d_bf16(&tq64, a.q, D, a.hq, a.num_tokens, 64, 64) ||
-          !encode_tma_3d_bf16(&tdo64, dout, D, a.hq, a.num_tokens, 64, 64) ||
-          !encode_tma_3d_f32(&tdq, dq_acc, D, a.hq, a.num_tokens, D, 64))
-        return cudaErrorInvalidValue;
       // the warpgroups' setmaxnreg targets are served from the registers the
       // block is launched with: refuse to launch a build that got fewer
       static int regs_ok = -1;
@@ -911,11 +868,13 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
         regs_ok = fa.numRegs == D128::REG_LAUNCH ? 1 : 0;
       }
       if (!regs_ok) return cudaErrorInvalidConfiguration;
+      alignas(64) CUtensorMap tdq32;  // fp32 accumulator, [128 rows][32 dims] boxes, 128-byte swizzle
+      if (!encode_tma_3d_f32(&tdq32, dq_acc, D, a.hq, a.num_tokens, 32, 128, true)) return cudaErrorInvalidValue;
       cudaError_t e = cudaFuncSetAttribute(bwd_main_d128, cudaFuncAttributeMaxDynamicSharedMemorySize, D128::SMEM);
       if (e != cudaSuccess) return e;
       bwd_main_d128<<<grid, D128::THREADS, D128::SMEM, st>>>(
-          tq64, tk, tv, tdo64, tdq, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv,
-          a.scale, a.scale * 1.4426950408889634f, lse, dvec, dq_acc, static_cast<__nv_bfloat16*>(dk),
+          tq, tk, tv, tdo, tdq32, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv,
+          a.scale, a.scale * 1.4426950408889634f, lse, dvec, static_cast<__nv_bfloat16*>(dk),
           static_cast<__nv_bfloat16*>(dv), a.status);
     } else {
       cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);

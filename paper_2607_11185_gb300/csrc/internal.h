@@ -64,9 +64,10 @@ cudaError_t launch_attn_bwd(const AttnArgs& a, const void* o, const float* lse, 
 bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d, uint64_t heads, uint64_t tokens,
                         uint32_t box_d, uint32_t box_rows);
 
-// fp32 variant without swizzle (bulk reduce-add targets).
+// fp32 variant (bulk reduce-add targets): no swizzle, or the 128-byte swizzle
+// (box_d * 4 must then be 128).
 bool encode_tma_3d_f32(void* map, const void* base, uint64_t d, uint64_t heads, uint64_t tokens, uint32_t box_d,
-                       uint32_t box_rows);
+                       uint32_t box_rows, bool swizzle128 = false);
 
 constexpr size_t kWsHeader = 256;  // attention workspace header (status word first)
 
