@@ -447,7 +447,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // With a 64-query sub-tile and two streams (compute of one stream overlapping
 // the other's MMAs) the N = 64 MMAs held the backward 5% lower on the
 // long-horizon workload than this single stream of 128-query tiles.
-//   TMEM: dV [0,128), dK [128,256), S^T then dQ [256,384), dP^T then P^T [384,512)
+//   TMEM: dV [0,128), dK [128,256); S^T then dQ, and dP^T then P^T, in [256,384) and
+//         [384,512), swapping roles every tile so that S^T(u+1) can be computed while
+//         dQ(u) is drained
 //   smem: K, V (64 KB), 2-stage Q/dO ring (128 KB; a freed stage also stages dQ),
 //         dS^T (32 KB), row terms (1 KB)
 
@@ -477,7 +479,10 @@ struct D128 {
   static constexpr int OFF_ROW = OFF_DS + TILE;                // WG k: -lse*log2e [64], -D*scale [64]
   static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * 64 * 4;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
-  static constexpr int TM_DV = 0, TM_DK = 128, TM_S = 256, TM_P = 384;
+  static constexpr int TM_DV = 0, TM_DK = 128, TM_A = 256, TM_B = 384;
+  // tile u: S^T (later dQ) in TM_A for even u, TM_B for odd u; dP^T (later P^T) in the other
+  __device__ static uint32_t col_s(int u) { return (u & 1) ? TM_B : TM_A; }
+  __device__ static uint32_t col_p(int u) { return (u & 1) ? TM_A : TM_B; }
   static constexpr int REG_CTRL = 104, REG_COMPUTE = 176, REG_DRAIN = 56;
   static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
@@ -614,9 +619,10 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::BLOCK, 1024);
       for (int u = 0; ok && u < U; ++u) {
         const int stage = u % C::NST;
-        // S^T = K Q^T and dP^T = V dO^T: need Q/dO of u and the S^T columns back (dQ of u-1 drained)
-        if (!mbar_wait(&bars->qdo_full[stage], (u / C::NST) & 1) ||
-            (u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) || aborted_now()) {
+        const uint32_t cs = tmem + C::col_s(u), cp = tmem + C::col_p(u);
+        // S^T = K Q^T needs Q/dO of u; its columns held P^T of u-1, which dV(u-1), issued
+        // before, reads first (in-order execution), so it overlaps the drain of dQ(u-1).
+        if (!mbar_wait(&bars->qdo_full[stage], (u / C::NST) & 1) || aborted_now()) {
           ok = false;
           break;
         }
@@ -625,12 +631,18 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t o = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
-          tc_mma_ss(tmem + C::TM_S, desc_at(k_kmaj, o), desc_at(qd, o), C::IDESC_S, kk > 0);
+          tc_mma_ss(cs, desc_at(k_kmaj, o), desc_at(qd, o), C::IDESC_S, kk > 0);
         }
+        // dP^T = V dO^T goes where dQ(u-1) was: wait for the drain to have read it
+        if (u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t o = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
-          tc_mma_ss(tmem + C::TM_P, desc_at(v_kmaj, o), desc_at(dd, o), C::IDESC_S, kk > 0);
+          tc_mma_ss(cp, desc_at(v_kmaj, o), desc_at(dd, o), C::IDESC_S, kk > 0);
         }
         tc_commit(&bars->s_full);
         // dQ = dS K, dV += P^T dO, dK += dS^T Q.  In-order execution keeps S(u+1) from
@@ -644,11 +656,11 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         const uint32_t acc0 = u > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < C::BM / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_S, desc_at(ds_mnmaj, kk * 2048), desc_at(k_mnmaj, kk * 2048), C::IDESC_DQ,
+          tc_mma_ss(cs, desc_at(ds_mnmaj, kk * 2048), desc_at(k_mnmaj, kk * 2048), C::IDESC_DQ,
                     kk > 0 ? 1u : 0u);
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ts(tmem + C::TM_DV, tmem + C::TM_P + (kk >> 2) * 64 + (kk & 3) * 8, desc_at(dmn, kk * 2048),
+          tc_mma_ts(tmem + C::TM_DV, cp + (kk >> 2) * 64 + (kk & 3) * 8, desc_at(dmn, kk * 2048),
                     C::IDESC_KV, kk > 0 ? 1u : acc0);
 #pragma unroll
         for (int kk = 0; kk < C::BQ / 16; ++kk)
@@ -697,10 +709,11 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       if (!mbar_wait(&bars->s_full, u & 1)) { ok = false; break; }
       tc_fence_after();
       uint32_t sv[64], pv[64];
-      tmem_ld_32x32b_x32(trow + C::TM_S + 64 * k, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-      tmem_ld_32x32b_x32(trow + C::TM_S + 64 * k + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
-      tmem_ld_32x32b_x32(trow + C::TM_P + 64 * k, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
-      tmem_ld_32x32b_x32(trow + C::TM_P + 64 * k + 32, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
+      const uint32_t cs = trow + C::col_s(u) + 64 * k, cp = trow + C::col_p(u) + 64 * k;
+      tmem_ld_32x32b_x32(cs, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
+      tmem_ld_32x32b_x32(cs + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
+      tmem_ld_32x32b_x32(cp, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
+      tmem_ld_32x32b_x32(cp + 32, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
       tmem_ld_wait();
       reg_fence<64>(sv);
       reg_fence<64>(pv);
@@ -730,7 +743,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         }
         st_shared_v4(ds_row + (uint32_t)((ch ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
       }
-      tmem_st_32x32b_x32(trow + C::TM_P + 64 * k, pt);   // P^T over this warpgroup's dP^T columns
+      tmem_st_32x32b_x32(cp, pt);                      // P^T over this warpgroup's dP^T columns
       tmem_st_wait();
       fence_proxy_async_smem();
       tc_fence_before();
@@ -789,7 +802,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
 #pragma unroll
       for (int part = 0; part < D / 32; ++part) {
         uint32_t a[32];
-        tmem_ld_32x32b_x32(trow + C::TM_S + part * 32, a);
+        tmem_ld_32x32b_x32(trow + C::col_s(u) + part * 32, a);
         tmem_ld_wait();
         reg_fence<32>(a);
         if (part == D / 32 - 1) {
