@@ -462,6 +462,8 @@ __device__ __forceinline__ void tma_reduce_add_3d(const void* map, const void* s
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// all but the most recent bulk group have finished reading their shared-memory sources
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 struct D128 {
@@ -495,9 +497,11 @@ static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D1
 
 struct D128Bars {
   uint64_t kv_full;
-  uint64_t qdo_full[D128::NST];
+  uint64_t q_full[D128::NST];      // Q of the stage's tile has landed
+  uint64_t do_full[D128::NST];     // dO of the stage's tile has landed
   uint64_t kv_done[D128::NST];     // the tile's MMAs are complete: its Q/dO stage may be overwritten
-  uint64_t stage_free[D128::NST];  // the drain's reduce-adds have read the stage
+  uint64_t q_free[D128::NST];      // the drain's reduce-adds have read the stage's Q half
+  uint64_t do_free[D128::NST];     // ... and its dO half
   uint64_t s_full;
   uint64_t p_full;
   uint64_t tmem_free;
@@ -550,9 +554,11 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   if (threadIdx.x == 0) {
     mbar_init(&bars->kv_full, 1);
     for (int i = 0; i < C::NST; ++i) {
-      mbar_init(&bars->qdo_full[i], 1);
+      mbar_init(&bars->q_full[i], 1);
+      mbar_init(&bars->do_full[i], 1);
       mbar_init(&bars->kv_done[i], 1);
-      mbar_init(&bars->stage_free[i], 1);
+      mbar_init(&bars->q_free[i], 1);
+      mbar_init(&bars->do_free[i], 1);
     }
     mbar_init(&bars->s_full, 1);
     mbar_init(&bars->p_full, 256);
@@ -593,18 +599,25 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         const int h = head_of(u);
         const int q0 = n * C::BM + sub_of(u) * C::BQ;
         const int stage = u % C::NST;
-        if (u >= C::NST && !mbar_wait(&bars->stage_free[stage], ((u / C::NST) - 1) & 1)) {
+        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::TILE;
+        // Q and dO are refilled separately: the drain's reduce-adds read the Q half first
+        if (u >= C::NST && !mbar_wait(&bars->q_free[stage], ((u / C::NST) - 1) & 1)) {
           abort_now();
           break;
         }
         if (aborted_now()) break;
-        mbar_arrive_expect_tx(&bars->qdo_full[stage], 2 * C::TILE);
-        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::TILE;
+        mbar_arrive_expect_tx(&bars->q_full[stage], C::TILE);
 #pragma unroll
-        for (int kb = 0; kb < 2; ++kb) {
-          tma_load_3d(qs + kb * C::BLOCK, &tm_q, &bars->qdo_full[stage], kb * 64, h, start + q0);
-          tma_load_3d(qs + C::TILE + kb * C::BLOCK, &tm_do, &bars->qdo_full[stage], kb * 64, h, start + q0);
+        for (int kb = 0; kb < 2; ++kb)
+          tma_load_3d(qs + kb * C::BLOCK, &tm_q, &bars->q_full[stage], kb * 64, h, start + q0);
+        if (u >= C::NST && !mbar_wait(&bars->do_free[stage], ((u / C::NST) - 1) & 1)) {
+          abort_now();
+          break;
         }
+        mbar_arrive_expect_tx(&bars->do_full[stage], C::TILE);
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb)
+          tma_load_3d(qs + C::TILE + kb * C::BLOCK, &tm_do, &bars->do_full[stage], kb * 64, h, start + q0);
       }
     } else if (warp == 1 && lane == 0) {
       // ---------------------------------------------------------- MMA issuer
@@ -622,7 +635,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         const uint32_t cs = tmem + C::col_s(u), cp = tmem + C::col_p(u);
         // S^T = K Q^T needs Q/dO of u; its columns held P^T of u-1, which dV(u-1), issued
         // before, reads first (in-order execution), so it overlaps the drain of dQ(u-1).
-        if (!mbar_wait(&bars->qdo_full[stage], (u / C::NST) & 1) || aborted_now()) {
+        if (!mbar_wait(&bars->q_full[stage], (u / C::NST) & 1) || aborted_now()) {
           ok = false;
           break;
         }
@@ -634,7 +647,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           tc_mma_ss(cs, desc_at(k_kmaj, o), desc_at(qd, o), C::IDESC_S, kk > 0);
         }
         // dP^T = V dO^T goes where dQ(u-1) was: wait for the drain to have read it
-        if (u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) {
+        if ((u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) ||
+            !mbar_wait(&bars->do_full[stage], (u / C::NST) & 1)) {
           ok = false;
           break;
         }
@@ -819,12 +833,16 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       if (dw == 0) {
         const int h = head_of(u);
         const int q0 = n * C::BM + sub_of(u) * C::BQ;
+        // blocks 0, 1 sit in the Q half, 2, 3 in the dO half: release each half once read
 #pragma unroll
-        for (int part = 0; part < D / 32; ++part)
+        for (int part = 0; part < D / 32; ++part) {
           tma_reduce_add_3d(&tm_dq, stg + part * (128 * 128), part * 32, h, start + q0);
-        bulk_commit();
+          if (part == 1 || part == 3) bulk_commit();
+        }
+        bulk_wait_read1();
+        mbar_arrive(&bars->q_free[stage]);
         bulk_wait_read();
-        mbar_arrive(&bars->stage_free[stage]);
+        mbar_arrive(&bars->do_free[stage]);
       }
       if (aborted_now()) { ok = false; break; }
     }
