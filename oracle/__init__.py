@@ -2,7 +2,8 @@
 
 A plain, slow, obviously correct restatement of what the path computes,
 written from the paper (Sec. 3.4, Algorithm 1, App. C.1 "Trajectory
-Processing Algorithm") and from the definition of causal softmax attention.
+Processing Algorithm", the RL objective of App. C.2) and from the definition
+of causal softmax attention.
 Floating point is fp64 throughout.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py`` (its CPU
@@ -17,4 +18,4 @@ Parity status: every function here is pinned by ``tests/test_oracle_*.py``
 (hand-worked segmentations, closed forms, invariants, a library special case,
 finite differences).  No function is "parity unpinned".
 """
-from . import segments, attention, gather  # noqa: F401
+from . import segments, attention, gather, loss  # noqa: F401

@@ -1,0 +1,99 @@
+"""Token-level RL objective over segments, fp64 (test infrastructure).
+
+The segments Algorithm 1 emits are consumed by the RL objective of App. C.2
+(Eq. "RL objective" and the hyperparameter table): for task i and rollout j
+with group-relative advantage A_ij shared by every segment of that rollout,
+
+  L = - E_i E_j  sum_{s in S_ij} sum_{t in s, mask_t = 1}
+          min( rho_t A_ij, clip(rho_t, 1 - eps_l, 1 + eps_h) A_ij )
+      + lambda * KL(pi_theta || pi_ref),
+
+rho_t = pi_theta(a_t | x_<t) / pi_rollout(a_t | x_<t), asymmetric clipping
+eps_l = 0.2, eps_h = 0.28 (DAPO), a clip-ratio cap c = 3.0 and a KL weight
+lambda = 1e-4.  The paper gives no formula for the cap or the KL estimator and
+no normaliser beyond the expectations; this oracle reads them as follows (the
+same readings are listed in the design doc):
+
+  * cap: dual clipping for negative advantages, the objective of a token with
+    A < 0 is max(min(rho A, clip(rho) A), c A);
+  * KL: the per-token estimator exp(r) - r - 1 with r = log pi_ref - log pi_theta,
+    taken over the same trainable tokens as the policy term;
+  * the expectations are means over the batch's trajectories (tasks x
+    rollouts): L = (1/N_traj) sum_t mask_t ( -o_t + lambda k_t );
+  * group-relative advantage: (r - mean_g r) / (std_g r + eps) over the n
+    rollouts of each task, population standard deviation.
+
+Inputs are log-probabilities.  The branch of the clipped objective a token
+takes depends on rho_t; it is decided in the kernel's precision (float32,
+rho = exp(float32(logp - old_logp))) so that both sides take the same branch,
+and the values are then evaluated in fp64.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def group_advantage(rewards, group_size: int, eps: float = 1e-6):
+    """GRPO group-relative advantage (App. C.2): rewards are [num_groups * group_size],
+    grouped consecutively; returns (r - mean) / (std + eps) per element, fp64."""
+    r = np.asarray(rewards, dtype=np.float64).reshape(-1, group_size)
+    mean = r.mean(axis=1, keepdims=True)
+    std = np.sqrt(((r - mean) ** 2).mean(axis=1, keepdims=True))
+    return ((r - mean) / (std + eps)).reshape(-1)
+
+
+def token_traj(cu_seqlens, seg_traj):
+    """Trajectory index of every segment token (segments in order)."""
+    cu = np.asarray(cu_seqlens, dtype=np.int64)
+    st = np.asarray(seg_traj, dtype=np.int64)
+    return np.repeat(st, np.diff(cu))
+
+
+def _branch_rho(logp, old_logp):
+    """rho in the kernel's precision, for the branch decision only."""
+    d = np.asarray(logp, dtype=np.float32) - np.asarray(old_logp, dtype=np.float32)
+    return np.exp(d.astype(np.float32)).astype(np.float32)
+
+
+def grpo_loss(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_traj: int,
+              eps_low: float = 0.2, eps_high: float = 0.28, clip_cap: float = 3.0, kl_coef: float = 1e-4):
+    """Loss value and its gradient with respect to logp (both fp64).
+
+    logp, old_logp, ref_logp: [num_tokens] per segment token; mask: [num_tokens]
+    (1 = trainable); cu_seqlens / seg_traj: the builder's layout; adv: [num_traj].
+    Returns (loss, dlogp)."""
+    lp = np.asarray(logp, dtype=np.float64)
+    old = np.asarray(old_logp, dtype=np.float64)
+    ref = np.asarray(ref_logp, dtype=np.float64)
+    m = np.asarray(mask).astype(np.float64)
+    a = np.asarray(adv, dtype=np.float64)[token_traj(cu_seqlens, seg_traj)]
+    n = lp.shape[0]
+    rho32 = _branch_rho(logp, old_logp)
+    loss_terms = np.zeros(n)
+    grad = np.zeros(n)
+    lo, hi = 1.0 - eps_low, 1.0 + eps_high
+    for t in range(n):
+        if m[t] == 0.0:
+            continue
+        rho = np.exp(lp[t] - old[t])
+        A = a[t]
+        rb = float(rho32[t])
+        # policy objective o and do/dlogp (rho-dependent branch -> rho*A, constant branch -> 0)
+        if A >= 0.0:
+            if rb <= np.float32(hi):
+                o, g = rho * A, rho * A
+            else:
+                o, g = hi * A, 0.0
+        else:
+            if rb < np.float32(lo):
+                o, g = lo * A, 0.0
+            elif rb > np.float32(clip_cap):
+                o, g = clip_cap * A, 0.0
+            else:
+                o, g = rho * A, rho * A
+        r = ref[t] - lp[t]
+        k = np.exp(r) - r - 1.0
+        dk = 1.0 - np.exp(r)          # d k / d logp
+        loss_terms[t] = -o + kl_coef * k
+        grad[t] = (-g + kl_coef * dk) / num_traj
+    return float(loss_terms.sum() / num_traj), grad
