@@ -318,7 +318,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="traj16x50_w8", choices=list(workloads.WORKLOADS))
     ap.add_argument("--layout", default=None, choices=[None, *workloads.COMPARISON_LAYOUTS],
-                    help="lay the traj32_w3 draw out as one of the comparison layouts")
+                    help="lay the workload's draw out as one of the comparison layouts (window, keep)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

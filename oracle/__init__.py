@@ -18,4 +18,4 @@ Parity status: every function here is pinned by ``tests/test_oracle_*.py``
 (hand-worked segmentations, closed forms, invariants, a library special case,
 finite differences).  No function is "parity unpinned".
 """
-from . import segments, attention, gather, loss  # noqa: F401
+from . import segments, attention, gather, loss, stream  # noqa: F401

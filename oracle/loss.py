@@ -97,3 +97,29 @@ def grpo_loss(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_tra
         loss_terms[t] = -o + kl_coef * k
         grad[t] = (-g + kl_coef * dk) / num_traj
     return float(loss_terms.sum() / num_traj), grad
+
+
+def grpo_loss_vec(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_traj: int,
+                  eps_low: float = 0.2, eps_high: float = 0.28, clip_cap: float = 3.0, kl_coef: float = 1e-4):
+    """grpo_loss written with whole-array operations (same branches and values), for
+    batches too large for the per-token loop.  Returns (loss, dlogp)."""
+    lp = np.asarray(logp, dtype=np.float64)
+    old = np.asarray(old_logp, dtype=np.float64)
+    ref = np.asarray(ref_logp, dtype=np.float64)
+    m = np.asarray(mask) != 0
+    a = np.asarray(adv, dtype=np.float64)[token_traj(cu_seqlens, seg_traj)]
+    rho = np.exp(lp - old)
+    rb = _branch_rho(logp, old_logp)
+    lo, hi = 1.0 - eps_low, 1.0 + eps_high
+    pos = a >= 0.0
+    const_pos = rb > np.float32(hi)
+    const_lo = rb < np.float32(lo)
+    const_cap = rb > np.float32(clip_cap)
+    o = np.where(pos, np.where(const_pos, hi * a, rho * a),
+                 np.where(const_lo, lo * a, np.where(const_cap, clip_cap * a, rho * a)))
+    dobj = np.where(pos, np.where(const_pos, 0.0, rho * a), np.where(const_lo | const_cap, 0.0, rho * a))
+    r = ref - lp
+    k = np.exp(r) - r - 1.0
+    terms = np.where(m, -o + kl_coef * k, 0.0)
+    grad = np.where(m, (-dobj + kl_coef * (1.0 - np.exp(r))) / num_traj, 0.0)
+    return float(terms.sum() / num_traj), grad

@@ -58,15 +58,17 @@ WORKLOADS: Dict[str, Workload] = {
                              outlier_frac=0.05),
 }
 
-# The same draw as traj32_w3 laid out four ways through the same kernels:
-# (window, keep).  "stepwise" (one item per turn with the prior history as
-# text) coincides with a window of one screenshot; the paper's own K = delta
-# settings are added so that the layouts differ.
+# The same draw laid out several ways through the same kernels: (window,
+# keep).  "stepwise" (one item per turn with the prior history as text)
+# coincides with a window of one screenshot; the paper's own K = delta
+# settings are added so that the layouts differ, and its ScienceBoard setting
+# K = 8, delta = 5 (App. C.2) as a K != delta case.
 COMPARISON_LAYOUTS: Dict[str, Tuple[int, int]] = {
     "stepwise": (1, 0),
     "w5": (5, 0),
     "paper_k1": (1, 1),
     "paper_k5": (5, 5),
+    "paper_k8_d5": (5, 8),
 }
 
 
