@@ -208,6 +208,94 @@ vcs_status vcs_attn_bwd_noalloc(const void* q, const void* k, const void* v, con
                                 float softmax_scale, void* dq, void* dk, void* dv, int32_t* dev_status,
                                 void* stream);
 
+/* ------------------------------------------------------------------------
+ * Token-ID stream fields (App. C.1, Algorithm 1's (ids, mask, logp) stream).
+ * Response tokens enter a segment's stream as trainable tokens with their
+ * rollout log-probabilities; observation tokens and the re-tokenised history
+ * of a fresh stream enter with mask 0 and log-probability 0.  Over the
+ * segment layout, for segment token n:
+ *   ids[n]  = traj_ids[tok_gather[n]]
+ *   logp[n] = tok_loss_mask[n] ? traj_logp[tok_gather[n]] : 0
+ *   traj_ids   int32 [traj_tokens] device: the trajectories' token IDs
+ *   traj_logp  fp32 [traj_tokens] device: rollout log-probabilities of the
+ *              trajectories' tokens (read only for response tokens)
+ *   tok_gather, tok_loss_mask  from vcs_build_segments
+ *   ids, logp  int32 / fp32 [num_tokens] device (written)
+ *   dev_status int32 device word or NULL: VCS_ERR_DEVICE_CHECK when a gather
+ *              index is outside [0, traj_tokens) (that token gets 0, 0)
+ * Returns VCS_ERR_INVALID_ARG for a negative count or a null pointer,
+ * VCS_ERR_OVERFLOW for counts above INT32_MAX.
+ * ------------------------------------------------------------------------ */
+vcs_status vcs_stream_fields(const int32_t* traj_ids, const float* traj_logp, int64_t traj_tokens,
+                             const int32_t* tok_gather, const uint8_t* tok_loss_mask, int64_t num_tokens,
+                             int32_t* ids, float* logp, int32_t* dev_status, void* stream);
+
+/* vcs_compact_trainable: the indices n with tok_loss_mask[n] != 0, in
+ * increasing order (each response token of the batch appears exactly once,
+ * App. C.1).
+ *   idx        int32 [idx_capacity] device (written: the first min(count,
+ *              idx_capacity) entries)
+ *   count      int64 device, 1 value (written): the number of trainable tokens
+ *   ws         device workspace of vcs_compact_workspace_size(num_tokens) bytes,
+ *              256-byte aligned; its first int32 is the device status word
+ *              (VCS_ERR_CAPACITY when count > idx_capacity)
+ * Returns VCS_ERR_INVALID_ARG for negative counts or null pointers,
+ * VCS_ERR_WORKSPACE for a small or misaligned workspace. */
+size_t vcs_compact_workspace_size(int64_t num_tokens);
+
+vcs_status vcs_compact_trainable(const uint8_t* tok_loss_mask, int64_t num_tokens, int32_t* idx, int64_t idx_capacity,
+                                 int64_t* count, void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * RL objective over the segments (App. C.2, Eq. "RL objective" and the
+ * hyperparameter table: DAPO asymmetric clipping eps_l = 0.2, eps_h = 0.28,
+ * clip-ratio cap c = 3.0, KL weight lambda = 1e-4, group-relative advantage
+ * shared by every segment of a rollout, loss masks so that each response is
+ * optimised exactly once).  Readings where the paper gives no formula:
+ *   - the cap is dual clipping: a token with A < 0 contributes
+ *     max(min(rho A, clip(rho, 1-eps_l, 1+eps_h) A), c A);
+ *   - the KL term is the per-token estimate exp(r) - r - 1, r = ref_logp - logp,
+ *     over the same trainable tokens;
+ *   - the expectations over tasks and rollouts are a mean over trajectories:
+ *       loss = (1/num_traj) sum_t mask_t (-o_t + kl_coef k_t).
+ *
+ * vcs_grpo_loss: forward and backward in one pass.
+ *   logp, old_logp, ref_logp  fp32 [num_tokens] device, segment layout: the
+ *               token log-probabilities under the policy being trained, the
+ *               rollout policy and the reference policy
+ *   tok_loss_mask u8 [num_tokens] device (vcs_build_segments' loss mask)
+ *   cu_seqlens, seg_traj  the layout from vcs_build_segments
+ *   adv         fp32 [num_traj] device: advantage of each trajectory
+ *   loss        fp64 device, 1 value (written)
+ *   dlogp       fp32 [num_tokens] device or NULL: d loss / d logp (written;
+ *               zero for masked tokens)
+ *   ws          device workspace of vcs_grpo_loss_workspace_size(num_tokens)
+ *               bytes, 256-byte aligned; its first int32 is the device status
+ *               word (VCS_ERR_DEVICE_CHECK when a segment names a trajectory
+ *               outside [0, num_traj); that token is skipped)
+ * Per token the ratio rho = exp(logp - old_logp) and the branch are float32;
+ * the sum is accumulated in double in a fixed order (deterministic).
+ * Returns VCS_ERR_INVALID_ARG for negative counts, num_traj <= 0, a null
+ * pointer, eps_low outside [0,1), eps_high < 0, clip_cap <= 1 + eps_high or
+ * kl_coef < 0; VCS_ERR_WORKSPACE for a small or misaligned workspace.
+ * ------------------------------------------------------------------------ */
+size_t vcs_grpo_loss_workspace_size(int64_t num_tokens);
+
+vcs_status vcs_grpo_loss(const float* logp, const float* old_logp, const float* ref_logp,
+                         const uint8_t* tok_loss_mask, const int32_t* cu_seqlens, const int32_t* seg_traj,
+                         int64_t num_segments, int64_t num_tokens, const float* adv, int64_t num_traj, float eps_low,
+                         float eps_high, float clip_cap, float kl_coef, double* loss, float* dlogp, void* ws,
+                         size_t ws_bytes, void* stream);
+
+/* vcs_group_advantage: GRPO's group-relative advantage (App. C.2: computed
+ * over the n rollouts of each task).  rewards fp32 [num_groups * group_size]
+ * device, each group's rollouts consecutive; adv (same shape, written) =
+ * (r - mean) / (std + eps) per group, population standard deviation, computed
+ * in double.  Returns VCS_ERR_INVALID_ARG for num_groups < 0, group_size <= 0,
+ * eps < 0 or a null pointer. */
+vcs_status vcs_group_advantage(const float* rewards, int64_t num_groups, int32_t group_size, float eps, float* adv,
+                               void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -226,6 +226,72 @@ size_t vcs_attn_bwd_workspace_size(int32_t num_segments, int64_t num_tokens, int
   return attn_bwd_ws_bytes(a);
 }
 
+vcs_status vcs_stream_fields(const int32_t* traj_ids, const float* traj_logp, int64_t traj_tokens,
+                             const int32_t* tok_gather, const uint8_t* tok_loss_mask, int64_t num_tokens,
+                             int32_t* ids, float* logp, int32_t* dev_status, void* stream) {
+  if (traj_tokens < 0 || num_tokens < 0) return VCS_ERR_INVALID_ARG;
+  if (traj_tokens > INT32_MAX || num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
+  if (num_tokens > 0 && (traj_ids == nullptr || traj_logp == nullptr || tok_gather == nullptr ||
+                         tok_loss_mask == nullptr || ids == nullptr || logp == nullptr))
+    return VCS_ERR_INVALID_ARG;
+  if (launch_stream_fields(traj_ids, traj_logp, traj_tokens, tok_gather, tok_loss_mask, num_tokens, ids, logp,
+                           dev_status, as_stream(stream)) != cudaSuccess)
+    return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+size_t vcs_compact_workspace_size(int64_t num_tokens) { return compact_ws_bytes(num_tokens < 0 ? 0 : num_tokens); }
+
+vcs_status vcs_compact_trainable(const uint8_t* tok_loss_mask, int64_t num_tokens, int32_t* idx, int64_t idx_capacity,
+                                 int64_t* count, void* ws, size_t ws_bytes, void* stream) {
+  if (num_tokens < 0 || idx_capacity < 0 || count == nullptr) return VCS_ERR_INVALID_ARG;
+  if (num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
+  if (num_tokens > 0 && tok_loss_mask == nullptr) return VCS_ERR_INVALID_ARG;
+  if (idx_capacity > 0 && idx == nullptr) return VCS_ERR_INVALID_ARG;
+  if (ws == nullptr || ws_bytes < compact_ws_bytes(num_tokens) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return VCS_ERR_WORKSPACE;
+  if (launch_compact(tok_loss_mask, num_tokens, idx, idx_capacity, count, ws, as_stream(stream)) != cudaSuccess)
+    return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+size_t vcs_grpo_loss_workspace_size(int64_t num_tokens) {
+  return grpo_loss_ws_bytes(num_tokens < 0 ? 0 : num_tokens);
+}
+
+vcs_status vcs_grpo_loss(const float* logp, const float* old_logp, const float* ref_logp,
+                         const uint8_t* tok_loss_mask, const int32_t* cu_seqlens, const int32_t* seg_traj,
+                         int64_t num_segments, int64_t num_tokens, const float* adv, int64_t num_traj, float eps_low,
+                         float eps_high, float clip_cap, float kl_coef, double* loss, float* dlogp, void* ws,
+                         size_t ws_bytes, void* stream) {
+  if (num_segments < 0 || num_tokens < 0 || num_traj <= 0 || loss == nullptr) return VCS_ERR_INVALID_ARG;
+  if (num_tokens > INT32_MAX || num_segments > INT32_MAX || num_traj > INT32_MAX) return VCS_ERR_OVERFLOW;
+  if (!(eps_low >= 0.f && eps_low < 1.f) || !(eps_high >= 0.f) || !(clip_cap > 1.f + eps_high) ||
+      !(kl_coef >= 0.f))
+    return VCS_ERR_INVALID_ARG;
+  if (num_tokens > 0 && (logp == nullptr || old_logp == nullptr || ref_logp == nullptr || tok_loss_mask == nullptr ||
+                         cu_seqlens == nullptr || seg_traj == nullptr || adv == nullptr || num_segments == 0))
+    return VCS_ERR_INVALID_ARG;
+  if (ws == nullptr || ws_bytes < grpo_loss_ws_bytes(num_tokens) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return VCS_ERR_WORKSPACE;
+  // branch thresholds rounded once from double, as a float32 reading of 1 - eps_l, 1 + eps_h
+  const float lo = (float)(1.0 - (double)eps_low), hi = (float)(1.0 + (double)eps_high);
+  if (launch_grpo_loss(logp, old_logp, ref_logp, tok_loss_mask, cu_seqlens, seg_traj, (int32_t)num_segments,
+                       (int32_t)num_tokens, adv, (int32_t)num_traj, lo, hi, clip_cap, kl_coef, loss, dlogp, ws,
+                       as_stream(stream)) != cudaSuccess)
+    return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+vcs_status vcs_group_advantage(const float* rewards, int64_t num_groups, int32_t group_size, float eps, float* adv,
+                               void* stream) {
+  if (num_groups < 0 || group_size <= 0 || !(eps >= 0.f)) return VCS_ERR_INVALID_ARG;
+  if (num_groups > 0 && (rewards == nullptr || adv == nullptr)) return VCS_ERR_INVALID_ARG;
+  if (launch_group_advantage(rewards, num_groups, group_size, eps, adv, as_stream(stream)) != cudaSuccess)
+    return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
 vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void* o, const float* lse,
                         const void* dout, const int32_t* cu_seqlens, int32_t num_segments, int64_t num_tokens,
                         int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* dq,

@@ -60,6 +60,23 @@ size_t attn_bwd_ws_bytes(const AttnArgs& a);
 cudaError_t launch_attn_bwd(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
                             void* dv, void* ws, cudaStream_t st);
 
+// ---- RL objective over segments (loss.cu) ----
+size_t grpo_loss_ws_bytes(int64_t num_tokens);
+cudaError_t launch_grpo_loss(const float* logp, const float* old_logp, const float* ref_logp, const uint8_t* mask,
+                             const int32_t* cu_seqlens, const int32_t* seg_traj, int32_t num_segments,
+                             int32_t num_tokens, const float* adv, int32_t num_traj, float lo, float hi,
+                             float clip_cap, float kl_coef, double* loss, float* dlogp, void* ws, cudaStream_t st);
+cudaError_t launch_group_advantage(const float* rewards, int64_t num_groups, int32_t group_size, float eps,
+                                   float* adv, cudaStream_t st);
+
+// ---- token-ID stream fields and trainable-token compaction (stream.cu) ----
+cudaError_t launch_stream_fields(const int32_t* traj_ids, const float* traj_logp, int64_t traj_tokens,
+                                 const int32_t* tok_gather, const uint8_t* mask, int64_t num_tokens, int32_t* ids,
+                                 float* logp, int32_t* status, cudaStream_t st);
+size_t compact_ws_bytes(int64_t num_tokens);
+cudaError_t launch_compact(const uint8_t* mask, int64_t num_tokens, int32_t* idx, int64_t capacity, int64_t* count,
+                           void* ws, cudaStream_t st);
+
 // TMA descriptor encoding through the driver entry point (no libcuda link).
 bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d, uint64_t heads, uint64_t tokens,
                         uint32_t box_d, uint32_t box_rows);

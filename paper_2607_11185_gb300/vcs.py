@@ -60,9 +60,20 @@ _lib_bwd = _sig("vcs_attn_bwd", _i32,
 _lib_bwd_noalloc = _sig("vcs_attn_bwd_noalloc", _i32,
                         [_p, _p, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p, _p])
 
+_f64 = ctypes.c_double
+_lib_loss_ws = _sig("vcs_grpo_loss_workspace_size", _sz, [_i64])
+_lib_loss = _sig("vcs_grpo_loss", _i32,
+                 [_p, _p, _p, _p, _p, _p, _i64, _i64, _p, _i64, _f32, _f32, _f32, _f32, _p, _p, _p, _sz, _p])
+_lib_adv = _sig("vcs_group_advantage", _i32, [_p, _i64, _i32, _f32, _p, _p])
+_lib_fields = _sig("vcs_stream_fields", _i32, [_p, _p, _i64, _p, _p, _i64, _p, _p, _p, _p])
+_lib_compact_ws = _sig("vcs_compact_workspace_size", _sz, [_i64])
+_lib_compact = _sig("vcs_compact_trainable", _i32, [_p, _i64, _p, _i64, _p, _p, _sz, _p])
+
 EXPORTED = ["vcs_status_string", "vcs_version", "vcs_segments_workspace_size", "vcs_plan_segments",
             "vcs_build_segments", "vcs_gather", "vcs_attn_fwd_workspace_size", "vcs_attn_fwd",
-            "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc"]
+            "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc", "vcs_grpo_loss_workspace_size",
+            "vcs_grpo_loss", "vcs_group_advantage", "vcs_stream_fields", "vcs_compact_workspace_size",
+            "vcs_compact_trainable"]
 
 LIB_PATH = _LIB_PATH
 
@@ -163,6 +174,36 @@ def vcs_attn_bwd_noalloc(q, k, v, o, lse, dout, cu_seqlens, num_segments, num_to
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
+def vcs_grpo_loss_workspace_size(num_tokens: int) -> int:
+    return int(_lib_loss_ws(num_tokens))
+
+
+def vcs_grpo_loss(logp, old_logp, ref_logp, tok_loss_mask, cu_seqlens, seg_traj, num_segments, num_tokens, adv,
+                  num_traj, eps_low, eps_high, clip_cap, kl_coef, loss, dlogp, ws, ws_bytes, stream=None) -> int:
+    return _lib_loss(_ptr(logp), _ptr(old_logp), _ptr(ref_logp), _ptr(tok_loss_mask), _ptr(cu_seqlens),
+                     _ptr(seg_traj), num_segments, num_tokens, _ptr(adv), num_traj, eps_low, eps_high, clip_cap,
+                     kl_coef, _ptr(loss), _ptr(dlogp), _ptr(ws), ws_bytes, _stream(stream))
+
+
+def vcs_group_advantage(rewards, num_groups, group_size, eps, adv, stream=None) -> int:
+    return _lib_adv(_ptr(rewards), num_groups, group_size, eps, _ptr(adv), _stream(stream))
+
+
+def vcs_stream_fields(traj_ids, traj_logp, traj_tokens, tok_gather, tok_loss_mask, num_tokens, ids, logp,
+                      dev_status, stream=None) -> int:
+    return _lib_fields(_ptr(traj_ids), _ptr(traj_logp), traj_tokens, _ptr(tok_gather), _ptr(tok_loss_mask),
+                       num_tokens, _ptr(ids), _ptr(logp), _ptr(dev_status), _stream(stream))
+
+
+def vcs_compact_workspace_size(num_tokens: int) -> int:
+    return int(_lib_compact_ws(num_tokens))
+
+
+def vcs_compact_trainable(tok_loss_mask, num_tokens, idx, idx_capacity, count, ws, ws_bytes, stream=None) -> int:
+    return _lib_compact(_ptr(tok_loss_mask), num_tokens, _ptr(idx), idx_capacity, _ptr(count), _ptr(ws), ws_bytes,
+                        _stream(stream))
+
+
 # ---------------------------------------------------------------- conveniences
 
 def _check(status: int, where: str):
@@ -258,6 +299,58 @@ def attn_bwd(q, k, v, o, lse, dout, cu_seqlens, max_seqlen: int, softmax_scale: 
     if check:
         _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_bwd (device)")
     return dq, dk, dv
+
+
+def grpo_loss(logp, old_logp, ref_logp, tok_loss_mask, cu_seqlens, seg_traj, adv, eps_low: float = 0.2,
+              eps_high: float = 0.28, clip_cap: float = 3.0, kl_coef: float = 1e-4, with_grad: bool = True,
+              stream=None, check=True):
+    """Loss (fp64 device scalar) and d loss / d logp (fp32, or None)."""
+    nt = logp.numel()
+    dev = logp.device
+    loss = torch.empty(1, dtype=torch.float64, device=dev)
+    dlogp = torch.empty(nt, dtype=torch.float32, device=dev) if with_grad else None
+    nb = vcs_grpo_loss_workspace_size(nt)
+    ws = _ws(nb, dev)
+    _check(vcs_grpo_loss(logp, old_logp, ref_logp, tok_loss_mask, cu_seqlens, seg_traj, seg_traj.numel(), nt, adv,
+                         adv.numel(), eps_low, eps_high, clip_cap, kl_coef, loss, dlogp, ws, nb, stream),
+           "vcs_grpo_loss")
+    if check:
+        _check(int(ws[:4].view(torch.int32).item()), "vcs_grpo_loss (device)")
+    return loss, dlogp
+
+
+def stream_fields(traj_ids, traj_logp, tok_gather, tok_loss_mask, stream=None):
+    """(ids int32, logp fp32) of every segment token (Algorithm 1's stream fields)."""
+    nt = tok_gather.numel()
+    dev = tok_gather.device
+    ids = torch.empty(nt, dtype=torch.int32, device=dev)
+    logp = torch.empty(nt, dtype=torch.float32, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    _check(vcs_stream_fields(traj_ids, traj_logp, traj_ids.numel(), tok_gather, tok_loss_mask, nt, ids, logp, status,
+                             stream), "vcs_stream_fields")
+    _check(int(status.item()), "vcs_stream_fields (device)")
+    return ids, logp
+
+
+def compact_trainable(tok_loss_mask, capacity=None, stream=None):
+    """Indices of the trainable tokens in order (int32 device tensor)."""
+    nt = tok_loss_mask.numel()
+    dev = tok_loss_mask.device
+    cap = nt if capacity is None else capacity
+    idx = torch.empty(max(cap, 1), dtype=torch.int32, device=dev)
+    count = torch.zeros(1, dtype=torch.int64, device=dev)
+    nb = vcs_compact_workspace_size(nt)
+    ws = _ws(nb, dev)
+    _check(vcs_compact_trainable(tok_loss_mask, nt, idx, cap, count, ws, nb, stream), "vcs_compact_trainable")
+    _check(int(ws[:4].view(torch.int32).item()), "vcs_compact_trainable (device)")
+    return idx[: int(count.item())]
+
+
+def group_advantage(rewards, group_size: int, eps: float = 1e-6, stream=None):
+    adv = torch.empty_like(rewards)
+    _check(vcs_group_advantage(rewards, rewards.numel() // group_size, group_size, eps, adv, stream),
+           "vcs_group_advantage")
+    return adv
 
 
 def default_scale(d: int) -> float:
