@@ -321,6 +321,7 @@ def main():
                     help="lay the workload's draw out as one of the comparison layouts (window, keep)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-next-rows", action="store_true", help="skip the stream-field / loss kernel timings")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -397,6 +398,8 @@ def main():
     if not args.no_e2e:
         e2e = run_e2e(path, args, flops * world, stream)
 
+    next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
+
     ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
     line = {
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -421,6 +424,7 @@ def main():
                      else None},
         "cpu_baseline": cpu,
         "e2e": e2e,
+        "next_rows": next_rows,
         "gpu_launches": path.launches_per_step * args.steps,
         "clocks": ck,
     }
@@ -428,6 +432,65 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
+
+
+def run_next_rows(path, stream, hbm_gbs):
+    """The stream fields, trainable-token compaction and RL objective (App. C.1-C.2) on the
+    largest chunk's layout, each launch timed alone with L2 flushed before it (CUDA events on
+    the launching stream, 3 warm-up + 10 timed launches).  HBM-bound: algorithmic bytes / time."""
+    vcs, w = path.vcs, path.w
+    ci = path.chunk_in[0]
+    lay = vcs.build_segments(ci["cu"], ci["img"], ci["txt"], path.window, path.keep, stream=stream)
+    nt, ntraj = lay["num_tokens"], ci["b1"] - ci["b0"]
+    ttok = ci["ttok1"] - ci["ttok0"]
+    gen = torch.Generator(path.dev).manual_seed(w.seed + 300)
+    traj_ids = torch.randint(0, 150000, (ttok,), generator=gen, device=path.dev, dtype=torch.int32)
+    traj_lp = -torch.rand(ttok, generator=gen, device=path.dev) * 6
+    ids = torch.empty(nt, dtype=torch.int32, device=path.dev)
+    old = torch.empty(nt, dtype=torch.float32, device=path.dev)
+    status = torch.zeros(1, dtype=torch.int32, device=path.dev)
+    logp = -torch.rand(nt, generator=gen, device=path.dev) * 6
+    ref = logp + torch.randn(nt, generator=gen, device=path.dev) * 0.1
+    adv = torch.randn(ntraj, generator=gen, device=path.dev)
+    loss = torch.empty(1, dtype=torch.float64, device=path.dev)
+    dlogp = torch.empty(nt, dtype=torch.float32, device=path.dev)
+    lws_bytes = vcs.vcs_grpo_loss_workspace_size(nt)
+    lws = torch.empty(max(lws_bytes, 256), dtype=torch.uint8, device=path.dev)
+    idx = torch.empty(nt, dtype=torch.int32, device=path.dev)
+    count = torch.zeros(1, dtype=torch.int64, device=path.dev)
+    cws_bytes = vcs.vcs_compact_workspace_size(nt)
+    cws = torch.empty(max(cws_bytes, 256), dtype=torch.uint8, device=path.dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=path.dev)
+    sp = stream.cuda_stream
+    ntrain = int(lay["tok_loss_mask"].sum().item())
+    calls = {
+        "stream_fields": (lambda: vcs.vcs_stream_fields(traj_ids, traj_lp, ttok, lay["tok_gather"],
+                                                        lay["tok_loss_mask"], nt, ids, old, status, sp),
+                          nt * (4 + 1 + 4 + 4 + 4) + 4 * ntrain),
+        "compact_trainable": (lambda: vcs.vcs_compact_trainable(lay["tok_loss_mask"], nt, idx, nt, count, cws,
+                                                                cws_bytes, sp), nt * 1 + 4 * ntrain),
+        "grpo_loss": (lambda: vcs.vcs_grpo_loss(logp, old, ref, lay["tok_loss_mask"], lay["cu_seqlens"],
+                                                lay["seg_traj"], lay["num_segments"], nt, adv, ntraj, 0.2, 0.28, 3.0,
+                                                1e-4, loss, dlogp, lws, lws_bytes, sp), nt * (4 + 4 + 4 + 1 + 4)),
+    }
+    out = {"tokens": nt, "trainable_tokens": ntrain, "l2": "flushed (256 MB write) before every timed launch"}
+    for name, (fn, nbytes) in calls.items():
+        times = []
+        for i in range(13):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            st = fn()
+            e1.record(stream)
+            assert st == 0, (name, st)
+            if i >= 3:
+                times.append((e0, e1))
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in times)
+        gbs = nbytes / (ms / 1e3) / 1e9
+        out[name] = {"ms": ms, "bytes": int(nbytes), "gbs": gbs, "frac_of_hbm": gbs / hbm_gbs}
+    assert int(status.item()) == 0 and int(lws[:4].view(torch.int32).item()) == 0
+    return out
 
 
 def run_e2e(path, args, flops, stream):

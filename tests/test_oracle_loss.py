@@ -128,3 +128,14 @@ def test_token_trajectory_map_follows_the_builder():
     # every segment token's source step lies inside the trajectory the map names
     step_traj = np.repeat(np.arange(3), np.diff(cu_steps))
     assert np.array_equal(step_traj[lay["tok_src_step"]], tt)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_vectorised_form_equals_the_token_loop(seed):
+    logp, old, ref, mask, cu, st, adv, nt = _random_case(seed + 20)
+    # include tokens exactly on the branch points
+    old[:3] = logp[:3] - np.log(np.array([0.8, 1.28, 3.0]))
+    l1, g1 = oloss.grpo_loss(logp, old, ref, mask, cu, st, adv, nt, kl_coef=0.2)
+    l2, g2 = oloss.grpo_loss_vec(logp, old, ref, mask, cu, st, adv, nt, kl_coef=0.2)
+    assert l2 == pytest.approx(l1, rel=1e-12, abs=1e-14)
+    np.testing.assert_allclose(g2, g1, rtol=1e-12, atol=1e-15)
