@@ -61,14 +61,16 @@ WORKLOADS: Dict[str, Workload] = {
 # The same draw laid out several ways through the same kernels: (window,
 # keep).  "stepwise" (one item per turn with the prior history as text)
 # coincides with a window of one screenshot; the paper's own K = delta
-# settings are added so that the layouts differ, and its ScienceBoard setting
-# K = 8, delta = 5 (App. C.2) as a K != delta case.
+# settings are added so that the layouts differ, its ScienceBoard setting
+# K = 8, delta = 5 (App. C.2) as a K != delta case, and K = delta = 8 as the
+# paper-exact reading of the long-horizon workload's window.
 COMPARISON_LAYOUTS: Dict[str, Tuple[int, int]] = {
     "stepwise": (1, 0),
     "w5": (5, 0),
     "paper_k1": (1, 1),
     "paper_k5": (5, 5),
     "paper_k8_d5": (5, 8),
+    "paper_k8": (8, 8),
 }
 
 
