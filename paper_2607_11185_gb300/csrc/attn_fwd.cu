@@ -50,6 +50,10 @@ namespace {
 using namespace dev;
 
 constexpr int kThreads = 384;
+// registers per thread after rebalancing: the producer/MMA warpgroup gives up
+// what the two softmax warpgroups take (the block launches with 168)
+constexpr int kRegLaunch = 168, kRegCtrl = 80, kRegSoftmax = 208;
+static_assert(kRegCtrl + 2 * kRegSoftmax <= 3 * kRegLaunch, "setmaxnreg targets exceed the launch registers");
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
@@ -175,9 +179,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_base;
 
-  if (warp == 0) {
+  if (warp < 4) {
+    setmaxnreg_dec<kRegCtrl>();
+    if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
@@ -206,10 +211,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, &bars->kv_full[slot], kb * 64, g,
                            start + j * C::BN, keep_l2);
       }
-    }
-  } else if (warp == 1) {
+    } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
       bool ok = mbar_wait(&bars->q_full, 0);
       // descriptors built once; the issue loops only add compile-time offsets
       const uint64_t q0d = smem_desc(sbase + C::OFF_Q0, 16, 1024), q1d = desc_at(q0d, C::TILE);
@@ -271,8 +274,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) on_timeout(bars, status);
     }
-  } else if (warp >= 4) {
+  } else {
     // ------------------------------------------------------------ softmax
+    setmaxnreg_inc<kRegSoftmax>();
     const int wg = (warp - 4) >> 2;
     const int quad = warp & 3;
     const int r = quad * 32 + lane;  // query row within the tile
@@ -412,6 +416,16 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
       !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
       !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128))
     return cudaErrorInvalidValue;
+  // the warpgroups' setmaxnreg targets are served from the registers the block
+  // is launched with: refuse to launch a build that got a different count
+  static int regs_ok = -1;
+  if (regs_ok < 0) {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, attn_fwd_kernel<D>);
+    if (e != cudaSuccess) return e;
+    regs_ok = fa.numRegs == kRegLaunch ? 1 : 0;
+  }
+  if (!regs_ok) return cudaErrorInvalidConfiguration;
   cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   const int npairs = (a.max_seqlen + 2 * C::BM - 1) / (2 * C::BM);
