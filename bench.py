@@ -209,13 +209,16 @@ class Path:
         self.bwd_ws = T(self.bwd_ws_bytes, dt=torch.uint8)
         self.launches_per_step = 0
 
-    def step(self, tstream, ev=None):
-        """One pass of the hot path over all chunks; optional (fwd, bwd) event pairs appended to ev."""
+    def step(self, tstream, ev=None, before_chunk=None, after_chunk=None):
+        """One pass of the hot path over all chunks; optional per-chunk events appended to ev and
+        hooks called before a chunk's first launch and after its last one."""
         vcs, w = self.vcs, self.w
         stream = tstream.cuda_stream
         hq, hkv, d = w.hq, w.hkv, w.d
         launches = 0
-        for ci in self.chunk_in:
+        for i, ci in enumerate(self.chunk_in):
+            if before_chunk is not None:
+                before_chunk(i)
             nseg, ntok = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"]
             evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)] if ev is not None else None
             if evs:
@@ -257,6 +260,8 @@ class Path:
             if evs:
                 evs[5].record(tstream)
                 ev.append((evs, ci))
+            if after_chunk is not None:
+                after_chunk(i)
         self.launches_per_step = launches
 
     def device_status(self):
@@ -513,17 +518,44 @@ def run_e2e(path, args, flops, stream):
     except RuntimeError as e:
         return {"value": None, "unit": "TFLOP/s", "error": f"pinned staging failed: {e}"[:200]}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = 0
+    # Each step's inputs are copied from pinned host memory on a second stream, chunk by
+    # chunk: a chunk's copy for the next step starts once its launches of this step are done,
+    # so it overlaps the other chunk's compute; the compute of a chunk waits for its copy.
+    cs = torch.cuda.Stream(device=path.dev)
+    nch = len(path.chunk_in)
+    copied = [torch.cuda.Event() for _ in range(nch)]
+    done = [torch.cuda.Event() for _ in range(nch)]
+    state = {"step": 0}
+
+    def copy_chunk(i):
+        ci = path.chunk_in[i]
+        a, b, t0_, t1_ = ci["ttok0"], ci["ttok1"], ci["tok0"], ci["tok1"]
+        with torch.cuda.stream(cs):
+            path.q_traj[a:b].copy_(host["q"][a:b], non_blocking=True)
+            path.k_traj[a:b].copy_(host["k"][a:b], non_blocking=True)
+            path.v_traj[a:b].copy_(host["v"][a:b], non_blocking=True)
+            path.dout[t0_:t1_].copy_(host["do"][t0_:t1_], non_blocking=True)
+            copied[i].record(cs)
+
+    def before(i):
+        stream.wait_event(copied[i])
+
+    def after(i):
+        done[i].record(stream)
+        if state["step"] + 1 < args.steps:           # the next step's inputs for this chunk
+            cs.wait_event(done[i])
+            copy_chunk(i)
+
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
-    for _ in range(args.steps):
-        path.q_traj.copy_(host["q"], non_blocking=True)
-        path.k_traj.copy_(host["k"], non_blocking=True)
-        path.v_traj.copy_(host["v"], non_blocking=True)
-        path.dout.copy_(host["do"], non_blocking=True)
-        path.step(stream)
+    cs.wait_event(t0)
+    for i in range(nch):
+        copy_chunk(i)
+    for s_ in range(args.steps):
+        state["step"] = s_
+        path.step(stream, before_chunk=before, after_chunk=after)
         # result read back: the last chunk's log-sum-exp (the loss-side statistic)
         res.copy_(path.lse.view(-1)[: res.numel()], non_blocking=True)
     t1.record(stream)
