@@ -466,6 +466,44 @@ __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.w
 __device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
+// One compute thread's share of a half tile: key row r against 32 query columns.
+//   P^T  = 2^(S^T * scale*log2e - lse*log2e)     (zero where the key follows the query)
+//   dS^T = P^T * (dP^T - D) * scale
+// The row terms come as {-lse*log2e, -D*scale} of each column pair, one 16-byte load
+// {nl(c), nl(c+1), nd(c), nd(c+1)} per pair.  P^T goes to pt as bf16 pairs; dS^T to
+// 16-byte chunks CH0 .. CH0+3 of the thread's 128-byte row of the swizzled K-major
+// shared block.  The causal test is compiled
+// only into the diagonal instantiation (column c is masked when c < dlim), so the
+// off-diagonal tiles run a branch-free body the compiler can interleave.
+template <bool DIAG>
+__device__ __forceinline__ void d128_half_math(const uint32_t (&sv)[32], const uint32_t (&pv)[32], uint32_t (&pt)[16],
+                                               const float* rt, uint64_t sl2, uint64_t sc2, int dlim, uint32_t ds_row,
+                                               int ch0, int r) {
+#pragma unroll
+  for (int ch = 0; ch < 4; ++ch) {
+    uint32_t wd[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int c = ch * 8 + e * 2;
+      const float4 q = *reinterpret_cast<const float4*>(&rt[2 * c]);
+      float x0, x1;
+      f2unpack(ffma2(f2pack(__uint_as_float(sv[c]), __uint_as_float(sv[c + 1])), sl2, f2pack(q.x, q.y)), x0, x1);
+      float p0 = ex2(x0), p1 = ex2(x1);
+      if (DIAG) {
+        if (c < dlim) p0 = 0.f;
+        if (c + 1 < dlim) p1 = 0.f;
+      }
+      const uint64_t pp = f2pack(p0, p1);
+      const uint64_t t = ffma2(f2pack(__uint_as_float(pv[c]), __uint_as_float(pv[c + 1])), sc2, f2pack(q.z, q.w));
+      float d0, d1;
+      f2unpack(fmul2(pp, t), d0, d1);
+      pt[ch * 4 + e] = pack_bf16(p0, p1);
+      wd[e] = pack_bf16(d0, d1);
+    }
+    st_shared_v4(ds_row + (uint32_t)(((ch0 + ch) ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
+  }
+}
+
 struct D128 {
   static constexpr int D = 128;
   static constexpr int BM = 128;                 // key rows of the tile
@@ -478,7 +516,7 @@ struct D128 {
   static constexpr int OFF_V = TILE;
   static constexpr int OFF_Q = 2 * TILE;                       // stage s: Q at +s*2*TILE, dO at +TILE
   static constexpr int OFF_DS = OFF_Q + NST * 2 * TILE;        // dS^T [128 keys][128 queries], two 64-query blocks
-  static constexpr int OFF_ROW = OFF_DS + TILE;                // WG k: -lse*log2e [64], -D*scale [64]
+  static constexpr int OFF_ROW = OFF_DS + TILE;                // WG k: -lse*log2e, -D*scale of 64 queries
   static constexpr int OFF_BAR = OFF_ROW + 2 * 2 * 64 * 4;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;
   static constexpr int TM_DV = 0, TM_DK = 128, TM_A = 256, TM_B = 384;
@@ -503,7 +541,7 @@ struct D128Bars {
   uint64_t q_free[D128::NST];      // the drain's reduce-adds have read the stage's Q half
   uint64_t do_free[D128::NST];     // ... and its dO half
   uint64_t s_full;
-  uint64_t p_full;
+  uint64_t p_full[2];  // query columns [0,64) / [64,128) of the tile: P^T and dS^T written
   uint64_t tmem_free;
   uint64_t acc_done;
   uint32_t tmem_base;
@@ -561,7 +599,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       mbar_init(&bars->do_free[i], 1);
     }
     mbar_init(&bars->s_full, 1);
-    mbar_init(&bars->p_full, 256);
+    mbar_init(&bars->p_full[0], 256);
+    mbar_init(&bars->p_full[1], 256);
     mbar_init(&bars->tmem_free, 128);
     mbar_init(&bars->acc_done, 1);
     bars->abort = 0;
@@ -659,27 +698,38 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           tc_mma_ss(cp, desc_at(v_kmaj, o), desc_at(dd, o), C::IDESC_S, kk > 0);
         }
         tc_commit(&bars->s_full);
-        // dQ = dS K, dV += P^T dO, dK += dS^T Q.  In-order execution keeps S(u+1) from
-        // overwriting P^T or dS^T before these read them.
-        if (!mbar_wait(&bars->p_full, u & 1)) {
+        // dV += P^T dO and dK += dS^T Q over the first 64 queries as soon as they are
+        // written (overlapping the compute of the other 64), then dQ = dS K and the rest
+        // of dV, dK.  In-order execution keeps S(u+1) from overwriting P^T or dS^T first.
+        // P^T of queries [16kk, 16kk+16) sits at column 64(kk/4) + 32((kk/2)%2) + 8(kk%2).
+        const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::TILE), dmn = desc_at(qmn, C::TILE);
+        const uint32_t acc0 = u > 0 ? 1u : 0u;
+        auto issue_dvdk = [&](int kk0) {
+#pragma unroll
+          for (int kk = kk0; kk < kk0 + 4; ++kk)
+            tc_mma_ts(tmem + C::TM_DV, cp + (kk >> 2) * 64 + ((kk >> 1) & 1) * 32 + (kk & 1) * 8,
+                      desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+#pragma unroll
+          for (int kk = kk0; kk < kk0 + 4; ++kk)
+            tc_mma_ss(tmem + C::TM_DK, desc_at(ds_kmaj, (kk >> 2) * C::BLOCK + (kk & 3) * 32),
+                      desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+        };
+        if (!mbar_wait(&bars->p_full[0], u & 1)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::TILE), dmn = desc_at(qmn, C::TILE);
-        const uint32_t acc0 = u > 0 ? 1u : 0u;
+        issue_dvdk(0);
+        if (!mbar_wait(&bars->p_full[1], u & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < C::BM / 16; ++kk)
           tc_mma_ss(cs, desc_at(ds_mnmaj, kk * 2048), desc_at(k_mnmaj, kk * 2048), C::IDESC_DQ,
                     kk > 0 ? 1u : 0u);
-#pragma unroll
-        for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ts(tmem + C::TM_DV, cp + (kk >> 2) * 64 + (kk & 3) * 8, desc_at(dmn, kk * 2048),
-                    C::IDESC_KV, kk > 0 ? 1u : acc0);
-#pragma unroll
-        for (int kk = 0; kk < C::BQ / 16; ++kk)
-          tc_mma_ss(tmem + C::TM_DK, desc_at(ds_kmaj, (kk >> 2) * C::BLOCK + (kk & 3) * 32),
-                    desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+        issue_dvdk(4);
         tc_commit(&bars->kv_done[stage]);
       }
       tc_commit(&bars->acc_done);
@@ -688,21 +738,22 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   } else if (warp < 12) {
     // ------------------------------------------------------------ compute
     setmaxnreg_inc<C::REG_COMPUTE>();
-    const int k = (warp - 4) >> 2;   // query columns [64k, 64k+64) of the tile
+    const int k = (warp - 4) >> 2;   // query columns [32k, 32k+32) and [64+32k, 96+32k) of the tile
     const int quad = warp & 3;
     const int r = quad * 32 + lane;  // TMEM lane: key row
     const int tw = threadIdx.x - 128 - k * 128;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    float* nl2_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;   // -lse*log2e per query
-    float* nds_s = nl2_s + 64;                                              // -D*scale per query
-    const uint32_t ds_row = sbase + C::OFF_DS + k * C::BLOCK + r * 128;
+    // row terms of the warpgroup's 64 query columns, per half of 32: {nl(c), nl(c+1), nd(c), nd(c+1)}
+    // for each column pair, nl = -lse*log2e and nd = -D*scale
+    float* rt_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;
+    const int rt_slot = (tw >> 5) * 64 + ((tw & 31) >> 1) * 4 + (tw & 1);  // this thread's column (tw < 64)
     const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
     auto row_terms = [&](int u, float& nl2, float& nds) {
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
       nds = 0.f;
       if (u < U && tw < 64) {
         const int h = head_of(u);
-        const int q = n * C::BM + sub_of(u) * C::BQ + 64 * k + tw;
+        const int q = n * C::BM + sub_of(u) * C::BQ + (tw < 32 ? 32 * k + tw : 32 + 32 * k + tw);
         if (q < L) {
           nl2 = -__ldg(&lse[(size_t)h * num_tokens + start + q]) * 1.4426950408889634f;
           nds = -__ldg(&dvec[(size_t)h * num_tokens + start + q]) * scale;
@@ -713,55 +764,37 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     row_terms(0, next_nl2, next_nds);
     bool ok = true;
     for (int u = 0; u < U; ++u) {
-      const int qoff = sub_of(u) * C::BQ + 64 * k;  // first query column of this warpgroup, from the key tile's first row
+      const bool diag = sub_of(u) == 0;  // the query rows are the key tile's own: mask keys after queries
       if (tw < 64) {
-        nl2_s[tw] = next_nl2;
-        nds_s[tw] = next_nds;
+        rt_s[rt_slot] = next_nl2;
+        rt_s[rt_slot + 2] = next_nds;
       }
       named_bar_sync(1 + k, 128);
       row_terms(u + 1, next_nl2, next_nds);
       if (!mbar_wait(&bars->s_full, u & 1)) { ok = false; break; }
       tc_fence_after();
-      uint32_t sv[64], pv[64];
-      const uint32_t cs = trow + C::col_s(u) + 64 * k, cp = trow + C::col_p(u) + 64 * k;
-      tmem_ld_32x32b_x32(cs, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
-      tmem_ld_32x32b_x32(cs + 32, *reinterpret_cast<uint32_t(*)[32]>(&sv[32]));
-      tmem_ld_32x32b_x32(cp, *reinterpret_cast<uint32_t(*)[32]>(&pv[0]));
-      tmem_ld_32x32b_x32(cp + 32, *reinterpret_cast<uint32_t(*)[32]>(&pv[32]));
-      tmem_ld_wait();
-      reg_fence<64>(sv);
-      reg_fence<64>(pv);
-      const bool diag = qoff < C::BM;                // these columns overlap the key tile's rows
-      uint32_t pt[32];                               // P^T row r: bf16 pairs (queries 2j, 2j+1)
+      // half hf: query columns [64hf + 32k, 64hf + 32k + 32); its P^T (16 words) goes over the
+      // first 16 of its own dP^T columns, its dS^T into chunks 4k..4k+3 of shared block hf
 #pragma unroll
-      for (int ch = 0; ch < 8; ++ch) {
-        uint32_t wd[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int c = ch * 8 + e * 2;
-          const float2 nl = *reinterpret_cast<const float2*>(&nl2_s[c]);
-          const float2 nd = *reinterpret_cast<const float2*>(&nds_s[c]);
-          float x0, x1;
-          f2unpack(ffma2(f2pack(__uint_as_float(sv[c]), __uint_as_float(sv[c + 1])), sl2, f2pack(nl.x, nl.y)), x0, x1);
-          float p0 = ex2(x0), p1 = ex2(x1);
-          if (diag) {                                  // key after query: P = 0
-            if (r > qoff + c) p0 = 0.f;
-            if (r > qoff + c + 1) p1 = 0.f;
-          }
-          const uint64_t pp = f2pack(p0, p1);
-          const uint64_t t = ffma2(f2pack(__uint_as_float(pv[c]), __uint_as_float(pv[c + 1])), sc2, f2pack(nd.x, nd.y));
-          float d0, d1;
-          f2unpack(fmul2(pp, t), d0, d1);
-          pt[ch * 4 + e] = pack_bf16(p0, p1);
-          wd[e] = pack_bf16(d0, d1);
-        }
-        st_shared_v4(ds_row + (uint32_t)((ch ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
+      for (int hf = 0; hf < 2; ++hf) {
+        const uint32_t col = 64 * hf + 32 * k;
+        uint32_t sv[32], pv[32], pt[16];
+        tmem_ld_32x32b_x32(trow + C::col_s(u) + col, sv);
+        tmem_ld_32x32b_x32(trow + C::col_p(u) + col, pv);
+        tmem_ld_wait();
+        reg_fence<32>(sv);
+        reg_fence<32>(pv);
+        const uint32_t ds_row = sbase + C::OFF_DS + hf * C::BLOCK + r * 128;
+        if (diag)
+          d128_half_math<true>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, r - (int)col, ds_row, 4 * k, r);
+        else
+          d128_half_math<false>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, 0, ds_row, 4 * k, r);
+        tmem_st_32x32b_x16(trow + C::col_p(u) + col, pt);
+        tmem_st_wait();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(&bars->p_full[hf]);
       }
-      tmem_st_32x32b_x32(cp, pt);                      // P^T over this warpgroup's dP^T columns
-      tmem_st_wait();
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(&bars->p_full);
       named_bar_sync(1 + k, 128);                      // everyone is done with this tile's row terms
       if (aborted_now()) { ok = false; break; }
     }
