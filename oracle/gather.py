@@ -14,3 +14,14 @@ def gather_rows(x, tok_gather):
         import torch
         return x.detach().cpu()[torch.from_numpy(idx)]
     return np.asarray(x)[idx]
+
+
+def scatter_add_rows(x_seg, tok_gather, traj_tokens: int):
+    """Adjoint of gather_rows: out[t] = sum of x_seg[n] over the segment tokens n with
+    tok_gather[n] = t (zero for a trajectory token no segment copies).  The gradient of a
+    loss with respect to the trajectory rows is this sum over the token's copies (the
+    chain rule through the copy); fp64."""
+    x = np.asarray(x_seg, dtype=np.float64)
+    out = np.zeros((int(traj_tokens),) + x.shape[1:], dtype=np.float64)
+    np.add.at(out, np.asarray(tok_gather, dtype=np.int64), x)
+    return out
