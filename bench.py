@@ -327,6 +327,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next-rows", action="store_true", help="skip the stream-field / loss kernel timings")
+    ap.add_argument("--no-fused", action="store_true", help="skip the gathered-attention (fused gather) timing")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -404,6 +405,7 @@ def main():
         e2e = run_e2e(path, args, flops * world, stream)
 
     next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
+    fused = None if args.no_fused else run_fused(path, stream)
 
     ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
     line = {
@@ -430,6 +432,7 @@ def main():
         "cpu_baseline": cpu,
         "e2e": e2e,
         "next_rows": next_rows,
+        "fused_gather": fused,
         "gpu_launches": path.launches_per_step * args.steps,
         "clocks": ck,
     }
@@ -495,6 +498,69 @@ def run_next_rows(path, stream, hbm_gbs):
         gbs = nbytes / (ms / 1e3) / 1e9
         out[name] = {"ms": ms, "bytes": int(nbytes), "gbs": gbs, "frac_of_hbm": gbs / hbm_gbs}
     assert int(status.item()) == 0 and int(lws[:4].view(torch.int32).item()) == 0
+    return out
+
+
+def run_fused(path, stream, reps=2):
+    """Attention reading Q/K/V straight from the trajectory tensors through the gather map
+    (vcs_attn_fwd_gathered / vcs_attn_bwd_gathered: no materialised copies, the backward's
+    gradients summed into trajectory layout) against gather + vcs_attn_fwd + vcs_attn_bwd, on
+    the largest chunk: 1 warm-up + `reps` timed passes each, CUDA events on the stream."""
+    vcs, w = path.vcs, path.w
+    hq, hkv, d = w.hq, w.hkv, w.d
+    ci = path.chunk_in[0]
+    sp = stream.cuda_stream
+    nseg, ntok, mx = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"], ci["max_seqlen"]
+    st = vcs.vcs_build_segments(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"], path.window,
+                                path.keep, path.max_seg, path.max_tok, path.cu_seqlens, None, path.tok_gather,
+                                path.tok_src, path.tok_pos, path.tok_mask, path.sizes, path.seg_ws,
+                                path.seg_ws_bytes, sp)
+    assert st == 0
+    ttok = ci["ttok1"] - ci["ttok0"]
+    qt, kt, vt = (x[ci["ttok0"]:ci["ttok1"]] for x in (path.q_traj, path.k_traj, path.v_traj))
+    dout = path.dout[ci["tok0"]:ci["tok1"]]
+    gws_bytes = vcs.vcs_attn_bwd_gathered_workspace_size(nseg, ntok, mx, ttok, hq, hkv, d)
+    gws = torch.empty(gws_bytes, dtype=torch.uint8, device=path.dev)
+    dqt, dkt, dvt = torch.empty_like(qt), torch.empty_like(kt), torch.empty_like(vt)
+    fl, f_fwd, f_bwd = credited_flops(path.seg_lens[ci["s0"]:ci["s1"]], hq, d)
+
+    # each a list of (part, launch) with events recorded between the parts
+    fused = [("fwd_ms", lambda: vcs.vcs_attn_fwd_gathered(qt, kt, vt, ttok, path.tok_gather, path.cu_seqlens, nseg,
+                                                          ntok, mx, hq, hkv, d, 0.0, path.o, path.lse, path.fwd_ws,
+                                                          path.fwd_ws_bytes, sp)),
+             ("bwd_ms", lambda: vcs.vcs_attn_bwd_gathered(qt, kt, vt, ttok, path.tok_gather, path.o, path.lse, dout,
+                                                          path.cu_seqlens, nseg, ntok, mx, hq, hkv, d, 0.0, dqt, dkt,
+                                                          dvt, gws, gws_bytes, sp))]
+    materialised = [("gather_ms", lambda: vcs.vcs_gather(qt, kt, vt, ttok, path.tok_gather, ntok, hq, hkv, d, path.q,
+                                                         path.k, path.v, path.gstatus, sp)),
+                    ("fwd_ms", lambda: vcs.vcs_attn_fwd(path.q, path.k, path.v, path.cu_seqlens, nseg, ntok, mx, hq,
+                                                        hkv, d, 0.0, path.o, path.lse, path.fwd_ws,
+                                                        path.fwd_ws_bytes, sp)),
+                    ("bwd_ms", lambda: vcs.vcs_attn_bwd(path.q, path.k, path.v, path.o, path.lse, dout,
+                                                        path.cu_seqlens, nseg, ntok, mx, hq, hkv, d, 0.0, path.dq,
+                                                        path.dk, path.dv, path.bwd_ws, path.bwd_ws_bytes, sp))]
+
+    out = {"chunk_segment_tokens": ntok, "chunk_trajectory_tokens": ttok}
+    for name, parts in (("fused", fused), ("materialised", materialised)):
+        runs = []
+        for i in range(1 + reps):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)]
+            e[0].record(stream)
+            for j, (_, fn) in enumerate(parts):
+                assert fn() == 0, (name, parts[j][0])
+                e[j + 1].record(stream)
+            if i > 0:
+                runs.append(e)
+        torch.cuda.synchronize()
+        ms = statistics.mean(e[0].elapsed_time(e[-1]) for e in runs)
+        out[name] = {"ms": ms, "tflops": fl / (ms / 1e3) / 1e12}
+        for j, (part, _) in enumerate(parts):
+            out[name][part] = statistics.mean(e[j].elapsed_time(e[j + 1]) for e in runs)
+    assert int(gws[:4].view(torch.int32).item()) == 0 and path.device_status() == (0, 0, 0)
+    out["fused"]["note"] = ("forward + backward with dQ, dK, dV scattered into trajectory layout "
+                            "(fp32 sums over each token's copies)")
+    out["materialised"]["note"] = "gather + forward + backward, gradients left in segment layout"
+    del gws, dqt, dkt, dvt
     return out
 
 

@@ -209,6 +209,54 @@ vcs_status vcs_attn_bwd_noalloc(const void* q, const void* k, const void* v, con
                                 void* stream);
 
 /* ------------------------------------------------------------------------
+ * Gathered attention: the forward and backward above, with Q, K and V read
+ * straight from the trajectory-layout tensors through the builder's gather
+ * map instead of from vcs_gather's segment-layout copies.  A segment holds
+ * copies of trajectory tokens (the text history re-tokenised into each fresh
+ * stream, Alg. 1, App. C.1; the screenshots kept across segments), so segment
+ * token n is trajectory token tok_gather[n]; the paper names no kernel for
+ * this, and these calls only fuse the copy into the attention's tile loads.
+ *
+ *   q_traj      bf16 [traj_tokens, hq, d] device, row-major
+ *   k_traj, v_traj  bf16 [traj_tokens, hkv, d] device
+ *   traj_tokens number of trajectory tokens (rows of the three tensors)
+ *   tok_gather  int32 [num_tokens] device, from vcs_build_segments; every
+ *               entry in [0, traj_tokens) (an entry outside is recorded as
+ *               VCS_ERR_DEVICE_CHECK in the workspace status word and read as
+ *               row 0)
+ *   cu_seqlens .. lse / dout   as for vcs_attn_fwd / vcs_attn_bwd (segment
+ *               layout: o, lse and dout have num_tokens rows; NULL allowed
+ *               when num_tokens is 0)
+ *   dq_traj     bf16 [traj_tokens, hq, d] device (written): the sum over the
+ *               segment copies n of trajectory token t (tok_gather[n] = t) of
+ *               dQ of copy n; dk_traj, dv_traj bf16 [traj_tokens, hkv, d]
+ *               likewise (tokens no segment reads get 0)
+ * The forward's o and lse equal vcs_attn_fwd's on vcs_gather's copies bit
+ * for bit.  The backward accumulates in fp32 (atomic adds, so the order of
+ * the additions and the last bits of dq, dk, dv vary from run to run) and
+ * needs the workspace vcs_attn_bwd_gathered_workspace_size() gives:
+ * vcs_attn_bwd's plus 4*traj_tokens*(hq + 2*hkv)*d bytes, each term rounded
+ * up to 256.  Errors as for vcs_attn_fwd / vcs_attn_bwd, plus
+ * VCS_ERR_INVALID_ARG for num_tokens > 0 with traj_tokens = 0 or a NULL
+ * tok_gather and VCS_ERR_OVERFLOW for traj_tokens above INT32_MAX.
+ * ------------------------------------------------------------------------ */
+vcs_status vcs_attn_fwd_gathered(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
+                                 const int32_t* tok_gather, const int32_t* cu_seqlens, int32_t num_segments,
+                                 int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
+                                 float softmax_scale, void* o, float* lse, void* ws, size_t ws_bytes,
+                                 void* stream);
+
+size_t vcs_attn_bwd_gathered_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                                            int64_t traj_tokens, int32_t hq, int32_t hkv, int32_t d);
+
+vcs_status vcs_attn_bwd_gathered(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
+                                 const int32_t* tok_gather, const void* o, const float* lse, const void* dout,
+                                 const int32_t* cu_seqlens, int32_t num_segments, int64_t num_tokens,
+                                 int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d, float softmax_scale,
+                                 void* dq_traj, void* dk_traj, void* dv_traj, void* ws, size_t ws_bytes,
+                                 void* stream);
+
+/* ------------------------------------------------------------------------
  * Token-ID stream fields (App. C.1, Algorithm 1's (ids, mask, logp) stream).
  * Response tokens enter a segment's stream as trainable tokens with their
  * rollout log-probabilities; observation tokens and the re-tokenised history

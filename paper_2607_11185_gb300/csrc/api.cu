@@ -61,6 +61,19 @@ bool encode_tma_3d_bf16(void* map, const void* base, uint64_t d, uint64_t heads,
   return r == CUDA_SUCCESS;
 }
 
+bool encode_tma_rows_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows) {
+  std::call_once(g_encode_once, load_encode_fn);
+  if (g_encode == nullptr) return false;
+  cuuint64_t dims[2] = {row_elems, rows > 0 ? rows : 1};
+  cuuint64_t strides[1] = {row_elems * 2};
+  cuuint32_t box[2] = {64, 1};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(static_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+                        dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool encode_tma_3d_f32(void* map, const void* base, uint64_t d, uint64_t heads, uint64_t tokens, uint32_t box_d,
                        uint32_t box_rows, bool swizzle128) {
   std::call_once(g_encode_once, load_encode_fn);
@@ -309,6 +322,83 @@ vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void*
   if (cudaMemsetAsync(ws, 0, kWsHeader, st) != cudaSuccess) return VCS_ERR_CUDA;
   if (num_tokens == 0 || num_segments == 0) return VCS_OK;
   if (launch_attn_bwd(a, o, lse, dout, dq, dk, dv, ws, st) != cudaSuccess) return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+// ---------------------------------------------------------------- gathered attention
+// The attention forward/backward reading Q, K, V straight from trajectory-layout tensors
+// through the builder's gather map (no materialised segment-layout copies); the backward
+// returns dQ, dK, dV in trajectory layout, the contributions of a token's copies summed.
+static vcs_status check_gathered(const AttnArgs& a, int64_t traj_tokens, const int32_t* tok_gather) {
+  vcs_status s = check_attn(a);
+  if (s != VCS_OK) return s;
+  if (traj_tokens < 0) return VCS_ERR_INVALID_ARG;
+  if (traj_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
+  if (a.num_tokens > 0 && (traj_tokens == 0 || tok_gather == nullptr)) return VCS_ERR_INVALID_ARG;
+  return VCS_OK;
+}
+
+vcs_status vcs_attn_fwd_gathered(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
+                                 const int32_t* tok_gather, const int32_t* cu_seqlens, int32_t num_segments,
+                                 int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
+                                 float softmax_scale, void* o, float* lse, void* ws, size_t ws_bytes, void* stream) {
+  AttnArgs a =
+      make_args(q_traj, k_traj, v_traj, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
+  vcs_status s = check_gathered(a, traj_tokens, tok_gather);
+  if (s != VCS_OK) return s;
+  a.tok_gather = tok_gather;
+  a.traj_tokens = traj_tokens;
+  if ((num_tokens > 0 && (o == nullptr || lse == nullptr)) || !aligned16(o) || !aligned16(lse))
+    return VCS_ERR_INVALID_ARG;  // o, lse may be NULL when there are no segment tokens
+  if (ws == nullptr || ws_bytes < attn_fwd_ws_bytes(a) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return VCS_ERR_WORKSPACE;
+  a.status = static_cast<int32_t*>(ws);
+  cudaStream_t st = as_stream(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, st) != cudaSuccess) return VCS_ERR_CUDA;
+  if (num_tokens == 0 || num_segments == 0) return VCS_OK;
+  if (launch_attn_fwd(a, o, lse, ws, st) != cudaSuccess) return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+size_t vcs_attn_bwd_gathered_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                                            int64_t traj_tokens, int32_t hq, int32_t hkv, int32_t d) {
+  AttnArgs a = make_args(nullptr, nullptr, nullptr, nullptr, num_segments, num_tokens, max_seqlen, hq, hkv, d, 0.f);
+  a.traj_tokens = traj_tokens;
+  return attn_bwd_ws_bytes(a);
+}
+
+vcs_status vcs_attn_bwd_gathered(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
+                                 const int32_t* tok_gather, const void* o, const float* lse, const void* dout,
+                                 const int32_t* cu_seqlens, int32_t num_segments, int64_t num_tokens,
+                                 int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d, float softmax_scale,
+                                 void* dq_traj, void* dk_traj, void* dv_traj, void* ws, size_t ws_bytes,
+                                 void* stream) {
+  AttnArgs a =
+      make_args(q_traj, k_traj, v_traj, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
+  vcs_status s = check_gathered(a, traj_tokens, tok_gather);
+  if (s != VCS_OK) return s;
+  a.tok_gather = tok_gather;
+  a.traj_tokens = traj_tokens;
+  const void* seg_ptrs[3] = {o, lse, dout};            // may be NULL when there are no segment tokens
+  const void* traj_ptrs[3] = {dq_traj, dk_traj, dv_traj};
+  for (const void* p : seg_ptrs)
+    if ((num_tokens > 0 && p == nullptr) || !aligned16(p)) return VCS_ERR_INVALID_ARG;
+  for (const void* p : traj_ptrs)
+    if ((traj_tokens > 0 && p == nullptr) || !aligned16(p)) return VCS_ERR_INVALID_ARG;
+  if (ws == nullptr || ws_bytes < attn_bwd_ws_bytes(a) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return VCS_ERR_WORKSPACE;
+  a.status = static_cast<int32_t*>(ws);
+  cudaStream_t st = as_stream(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, st) != cudaSuccess) return VCS_ERR_CUDA;
+  if (num_tokens == 0 || num_segments == 0) {  // no segment token reads the trajectory: zero gradients
+    const size_t qb = (size_t)traj_tokens * hq * d * 2, kb = (size_t)traj_tokens * hkv * d * 2;
+    if (traj_tokens > 0 && (cudaMemsetAsync(dq_traj, 0, qb, st) != cudaSuccess ||
+                            cudaMemsetAsync(dk_traj, 0, kb, st) != cudaSuccess ||
+                            cudaMemsetAsync(dv_traj, 0, kb, st) != cudaSuccess))
+      return VCS_ERR_CUDA;
+    return VCS_OK;
+  }
+  if (launch_attn_bwd(a, o, lse, dout, dq_traj, dk_traj, dv_traj, ws, st) != cudaSuccess) return VCS_ERR_CUDA;
   return VCS_OK;
 }
 

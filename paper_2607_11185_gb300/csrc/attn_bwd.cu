@@ -147,6 +147,25 @@ __global__ void __launch_bounds__(256) bwd_dq_cvt(const float* __restrict__ acc,
   }
 }
 
+// ------------------------------------------------------------------ bwd_dq_scatter
+// Gathered backward: dq_traj[tok_gather[n]] += dq_acc[n] (fp32, all heads of the row), one
+// 16-byte chunk per thread; a segment token's rows are contiguous, so consecutive threads
+// add to one trajectory row.
+__global__ void __launch_bounds__(256) bwd_dq_scatter(const float* __restrict__ dq_acc,
+                                                      const int32_t* __restrict__ tok_gather, int64_t num_tokens,
+                                                      int32_t row_chunks, int32_t traj_tokens,
+                                                      float* __restrict__ dq_traj) {
+  const int64_t total = num_tokens * row_chunks;
+  for (int64_t i = blockIdx.x * 256ll + threadIdx.x; i < total; i += (int64_t)gridDim.x * 256) {
+    const int64_t n = i / row_chunks;
+    const int c = (int)(i - n * row_chunks);
+    const int t = __ldg(&tok_gather[n]);
+    if (t < 0 || t >= traj_tokens) continue;  // recorded by the attention kernels' gathers
+    const float4 x = reinterpret_cast<const float4*>(dq_acc)[i];
+    red_add_v4(dq_traj + ((int64_t)t * row_chunks + c) * 4, x.x, x.y, x.z, x.w);
+  }
+}
+
 // ------------------------------------------------------------------ bwd_main
 template <int D>
 __device__ __forceinline__ void issue_st(uint32_t tmem_d, uint32_t a_addr, uint32_t b_addr) {
@@ -179,14 +198,22 @@ __device__ __forceinline__ void issue_dq(uint32_t tmem_d, uint32_t dst_addr, uin
   }
 }
 
-template <int D>
+// GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
+// tile (TMA gather4 with the 2-D maps tm_q/k/v, or tiled loads with the 3-D maps
+// tm_qr/kr/vr where a tile is one run of consecutive trajectory rows), and dK, dV are added
+// in fp32 to trajectory-layout accumulators (dk_acc, dv_acc) at row tok_gather[key];
+// otherwise segment-layout tiled loads, bf16 dK, dV, and tm_qr/kr/vr unused.
+template <int D, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     bwd_main(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
              const int32_t* __restrict__ cu_seqlens, int32_t num_segments, int32_t num_tokens, int32_t max_seqlen,
              int32_t hq, int32_t hkv, int32_t ntiles, float scale, float scale_log2,
              const float* __restrict__ lse, const float* __restrict__ dvec, float* __restrict__ dq_acc,
-             __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status) {
+             __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status,
+             const int32_t* __restrict__ tok_gather, int32_t traj_tokens, float* __restrict__ dk_acc,
+             float* __restrict__ dv_acc, const __grid_constant__ CUtensorMap tm_qr,
+             const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr) {
   using C = Bwd<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -241,7 +268,42 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
+    if constexpr (GATHER) {
+      // the whole warp gathers Q, K, V; lane 0 posts the bytes, waits for free stages, loads dO
+      if (lane == 0) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_v);
+        tma_prefetch_desc(&tm_do);
+        mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
+      }
+      __syncwarp();
+      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &bars->kv_full, g, D, start + n * C::BM, end - 1,
+                                   tok_gather, traj_tokens, status, lane);
+      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &bars->kv_full, g, D, start + n * C::BM, end - 1,
+                                   tok_gather, traj_tokens, status, lane);
+      for (int it = 0; it < iters; ++it) {
+        const int h = g * G + it / per_head;
+        const int m = n + it % per_head;
+        int go = 1;
+        if (lane == 0) {
+          if (it > 0 && !mbar_wait(&bars->qdo_empty, (it - 1) & 1)) {
+            on_timeout(bars, status);
+            go = 0;
+          } else if (aborted(bars)) {
+            go = 0;
+          } else {
+            mbar_arrive_expect_tx(&bars->qdo_full, 2 * C::TILE);
+#pragma unroll
+            for (int kb = 0; kb < C::KB; ++kb)
+              tma_load_3d(smem + C::OFF_DO + kb * C::BLOCK, &tm_do, &bars->qdo_full, kb * 64, h, start + m * C::BN);
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q, &tm_q, &tm_qr, &bars->qdo_full, h, D, start + m * C::BN, end - 1,
+                                     tok_gather, traj_tokens, status, lane);
+      }
+    } else if (lane == 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
       tma_prefetch_desc(&tm_v);
@@ -391,8 +453,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       on_timeout(bars, status);
     } else {
       // dK, dV rows of the tile (key rows on TMEM lanes), this warpgroup's D/2 columns
-      const bool valid = kpos < L;
-      const size_t base = ((size_t)(start + kpos) * hkv + g) * D + wg * (D / 2);
+      bool valid = kpos < L;
+      size_t base = ((size_t)(start + kpos) * hkv + g) * D + wg * (D / 2);
+      if (GATHER && valid) {  // fp32 add at the key's trajectory row
+        const int t = tok_gather[start + kpos];
+        valid = t >= 0 && t < traj_tokens;
+        base = ((size_t)(valid ? t : 0) * hkv + g) * D + wg * (D / 2);
+      }
 #pragma unroll
       for (int which = 0; which < 2; ++which) {
         const uint32_t col = (which == 0 ? C::TM_DK : C::TM_DV) + wg * (D / 2);
@@ -403,7 +470,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_32x32b_x32(trow + col + c * 32, v32);
           tmem_ld_wait();
           reg_fence<32>(v32);
-          if (valid) {
+          if (GATHER) {
+            if (valid) {
+              float* acc = (which == 0 ? dk_acc : dv_acc) + base + c * 32;
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+                red_add_v4(acc + e * 4, __uint_as_float(v32[e * 4]), __uint_as_float(v32[e * 4 + 1]),
+                           __uint_as_float(v32[e * 4 + 2]), __uint_as_float(v32[e * 4 + 3]));
+            }
+          } else if (valid) {
             uint4* d4 = reinterpret_cast<uint4*>(outp + c * 32);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -549,13 +624,19 @@ struct D128Bars {
 };
 
 
+// GATHER: as for bwd_main (Q, K, V gathered from trajectory-layout tensors, dK and dV
+// added in fp32 at the keys' trajectory rows).
+template <bool GATHER>
 __global__ void __launch_bounds__(D128::THREADS, 1)
     bwd_main_d128(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                   const __grid_constant__ CUtensorMap tm_dq, const int32_t* __restrict__ cu_seqlens,
                   int32_t num_segments, int32_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, float scale,
                   float scale_log2, const float* __restrict__ lse, const float* __restrict__ dvec,
-                  __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status) {
+                  __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status,
+                  const int32_t* __restrict__ tok_gather, int32_t traj_tokens, float* __restrict__ dk_acc,
+                  float* __restrict__ dv_acc, const __grid_constant__ CUtensorMap tm_qr,
+                  const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr) {
   using C = D128;
   constexpr int D = C::D;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -622,7 +703,55 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
 
   if (warp < 4) {
     setmaxnreg_dec<C::REG_CTRL>();
-    if (warp == 0 && lane == 0) {
+    if (GATHER && warp == 0) {
+      // ---------------------------------------------------------- producer (gathered)
+      // the whole warp gathers K, V and each tile's Q; lane 0 posts the bytes, waits for
+      // free stages and loads dO
+      if (lane == 0) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_v);
+        tma_prefetch_desc(&tm_do);
+        mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
+      }
+      __syncwarp();
+      load_traj_tile<2, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
+                               traj_tokens, status, lane);
+      load_traj_tile<2, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
+                               traj_tokens, status, lane);
+      for (int u = 0; u < U; ++u) {
+        const int h = head_of(u);
+        const int q0 = n * C::BM + sub_of(u) * C::BQ;
+        const int stage = u % C::NST;
+        uint8_t* qs = smem + C::OFF_Q + stage * 2 * C::TILE;
+        int go = 1;
+        if (lane == 0) {
+          if (u >= C::NST && !mbar_wait(&bars->q_free[stage], ((u / C::NST) - 1) & 1)) {
+            abort_now();
+            go = 0;
+          } else if (aborted_now()) {
+            go = 0;
+          } else {
+            mbar_arrive_expect_tx(&bars->q_full[stage], C::TILE);
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+        load_traj_tile<2, C::BLOCK>(qs, &tm_q, &tm_qr, &bars->q_full[stage], h, D, start + q0, end - 1, tok_gather, traj_tokens,
+                                 status, lane);
+        if (lane == 0) {
+          if (u >= C::NST && !mbar_wait(&bars->do_free[stage], ((u / C::NST) - 1) & 1)) {
+            abort_now();
+            go = 0;
+          } else {
+            mbar_arrive_expect_tx(&bars->do_full[stage], C::TILE);
+#pragma unroll
+            for (int kb = 0; kb < 2; ++kb)
+              tma_load_3d(qs + C::TILE + kb * C::BLOCK, &tm_do, &bars->do_full[stage], kb * 64, h, start + q0);
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+      }
+    } else if (warp == 0 && lane == 0) {
       // ---------------------------------------------------------- producer
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_k);
@@ -807,13 +936,25 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const int kpos = n * C::BM + r;
       const uint32_t col = k == 0 ? C::TM_DK : C::TM_DV;
       __nv_bfloat16* outp = (k == 0 ? dk : dv) + ((size_t)(start + kpos) * hkv + g) * D;
+      float* accp = nullptr;  // gathered: fp32 add at the key's trajectory row
+      if (GATHER && kpos < L) {
+        const int t = tok_gather[start + kpos];
+        if (t >= 0 && t < traj_tokens) accp = (k == 0 ? dk_acc : dv_acc) + ((size_t)t * hkv + g) * D;
+      }
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t v32[32];
         tmem_ld_32x32b_x32(trow + col + c * 32, v32);
         tmem_ld_wait();
         reg_fence<32>(v32);
-        if (kpos < L) {
+        if (GATHER) {
+          if (accp != nullptr) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              red_add_v4(accp + c * 32 + e * 4, __uint_as_float(v32[e * 4]), __uint_as_float(v32[e * 4 + 1]),
+                         __uint_as_float(v32[e * 4 + 2]), __uint_as_float(v32[e * 4 + 3]));
+          }
+        } else if (kpos < L) {
           uint4* d4 = reinterpret_cast<uint4*>(outp + c * 32);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
@@ -894,14 +1035,23 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
 
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-template <int D>
+template <int D, bool GATHER>
 cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
                          void* dv, void* ws, cudaStream_t st) {
   using C = Bwd<D>;
   char* w = static_cast<char*>(ws) + kWsHeader;
   float* dvec = reinterpret_cast<float*>(w);
   float* dq_acc = reinterpret_cast<float*>(w + align256((size_t)a.hq * a.num_tokens * 4));
+  // gathered: fp32 trajectory-layout accumulators of dQ, dK, dV after the segment-layout dQ
+  float* dq_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dq_acc) + align256((size_t)a.num_tokens * a.hq * D * 4));
+  float* dk_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dq_t) + align256((size_t)a.traj_tokens * a.hq * D * 4));
+  float* dv_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dk_t) + align256((size_t)a.traj_tokens * a.hkv * D * 4));
   const int64_t rows = a.num_tokens * a.hq;
+  if (GATHER) {
+    const size_t span = reinterpret_cast<char*>(dv_t) - reinterpret_cast<char*>(dq_t) +
+                        (size_t)a.traj_tokens * a.hkv * D * 4;  // dq_t .. end of dv_t
+    if (cudaMemsetAsync(dq_t, 0, span, st) != cudaSuccess) return cudaErrorUnknown;
+  }
   {
     const int64_t total = rows * (D / 8);
     int64_t blocks = (total + kPreThreads - 1) / kPreThreads;
@@ -910,12 +1060,21 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
                                                          static_cast<const __nv_bfloat16*>(dout), rows, a.hq,
                                                          a.num_tokens, dvec, dq_acc);
   }
-  alignas(64) CUtensorMap tq, tk, tv, tdo;
-  if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
-      !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
-      !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128) ||
-      !encode_tma_3d_bf16(&tdo, dout, D, a.hq, a.num_tokens, 64, 128))
+  alignas(64) CUtensorMap tq, tk, tv, tdo, tqr, tkr, tvr;
+  if (GATHER) {
+    if (!encode_tma_rows_bf16(&tq, a.q, (uint64_t)a.hq * D, a.traj_tokens) ||
+        !encode_tma_rows_bf16(&tk, a.k, (uint64_t)a.hkv * D, a.traj_tokens) ||
+        !encode_tma_rows_bf16(&tv, a.v, (uint64_t)a.hkv * D, a.traj_tokens) ||
+        !encode_tma_3d_bf16(&tqr, a.q, D, a.hq, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tkr, a.k, D, a.hkv, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128))
+      return cudaErrorInvalidValue;
+  } else if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
+             !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
+             !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128)) {
     return cudaErrorInvalidValue;
+  }
+  if (!encode_tma_3d_bf16(&tdo, dout, D, a.hq, a.num_tokens, 64, 128)) return cudaErrorInvalidValue;
   const int ntiles = (a.max_seqlen + C::BM - 1) / C::BM;
   const int64_t gx = (int64_t)a.num_segments * a.hkv;
   if (gx > (int64_t)65535 * 65535) return cudaErrorInvalidConfiguration;
@@ -927,34 +1086,51 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
       static int regs_ok = -1;
       if (regs_ok < 0) {
         cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, bwd_main_d128);
+        cudaError_t e = cudaFuncGetAttributes(&fa, bwd_main_d128<GATHER>);
         if (e != cudaSuccess) return e;
         regs_ok = fa.numRegs == D128::REG_LAUNCH ? 1 : 0;
       }
       if (!regs_ok) return cudaErrorInvalidConfiguration;
       alignas(64) CUtensorMap tdq32;  // fp32 accumulator, [128 rows][32 dims] boxes, 128-byte swizzle
       if (!encode_tma_3d_f32(&tdq32, dq_acc, D, a.hq, a.num_tokens, 32, 128, true)) return cudaErrorInvalidValue;
-      cudaError_t e = cudaFuncSetAttribute(bwd_main_d128, cudaFuncAttributeMaxDynamicSharedMemorySize, D128::SMEM);
+      cudaError_t e =
+          cudaFuncSetAttribute(bwd_main_d128<GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, D128::SMEM);
       if (e != cudaSuccess) return e;
-      bwd_main_d128<<<grid, D128::THREADS, D128::SMEM, st>>>(
+      bwd_main_d128<GATHER><<<grid, D128::THREADS, D128::SMEM, st>>>(
           tq, tk, tv, tdo, tdq32, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv,
           a.scale, a.scale * 1.4426950408889634f, lse, dvec, static_cast<__nv_bfloat16*>(dk),
-          static_cast<__nv_bfloat16*>(dv), a.status);
+          static_cast<__nv_bfloat16*>(dv), a.status, a.tok_gather, (int32_t)a.traj_tokens, dk_t, dv_t,
+          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv);
     } else {
-      cudaError_t e = cudaFuncSetAttribute(bwd_main<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+      cudaError_t e =
+          cudaFuncSetAttribute(bwd_main<D, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
       if (e != cudaSuccess) return e;
-      bwd_main<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, tdo, a.cu_seqlens, a.num_segments,
-                                                   (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles, a.scale,
-                                                   a.scale * 1.4426950408889634f, lse, dvec, dq_acc,
-                                                   static_cast<__nv_bfloat16*>(dk), static_cast<__nv_bfloat16*>(dv),
-                                                   a.status);
+      bwd_main<D, GATHER><<<grid, kThreads, C::SMEM, st>>>(
+          tq, tk, tv, tdo, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles,
+          a.scale, a.scale * 1.4426950408889634f, lse, dvec, dq_acc, static_cast<__nv_bfloat16*>(dk),
+          static_cast<__nv_bfloat16*>(dv), a.status, a.tok_gather, (int32_t)a.traj_tokens, dk_t, dv_t,
+          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv);
     }
   }
-  {
-    const int64_t n8 = rows * D / 8;
+  auto convert = [&](const float* acc, void* out, int64_t elems) {
+    const int64_t n8 = elems / 8;
     int64_t blocks = (n8 + 255) / 256;
     if (blocks > 152 * 32) blocks = 152 * 32;
-    if (n8 > 0) bwd_dq_cvt<<<(unsigned)blocks, 256, 0, st>>>(dq_acc, static_cast<__nv_bfloat16*>(dq), n8);
+    if (n8 > 0) bwd_dq_cvt<<<(unsigned)blocks, 256, 0, st>>>(acc, static_cast<__nv_bfloat16*>(out), n8);
+  };
+  if (GATHER) {
+    const int32_t row_chunks = a.hq * D / 4;
+    const int64_t total = a.num_tokens * row_chunks;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    if (total > 0)
+      bwd_dq_scatter<<<(unsigned)blocks, 256, 0, st>>>(dq_acc, a.tok_gather, a.num_tokens, row_chunks,
+                                                       (int32_t)a.traj_tokens, dq_t);
+    convert(dq_t, dq, a.traj_tokens * a.hq * D);
+    convert(dk_t, dk, a.traj_tokens * a.hkv * D);
+    convert(dv_t, dv, a.traj_tokens * a.hkv * D);
+  } else {
+    convert(dq_acc, dq, rows * D);
   }
   return cudaGetLastError();
 }
@@ -962,14 +1138,21 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
 }  // namespace
 
 size_t attn_bwd_ws_bytes(const AttnArgs& a) {
-  if (a.num_tokens < 0 || a.hq <= 0 || a.d <= 0) return kWsHeader;
-  return kWsHeader + align256((size_t)a.hq * a.num_tokens * 4) + align256((size_t)a.num_tokens * a.hq * a.d * 4);
+  if (a.num_tokens < 0 || a.hq <= 0 || a.hkv <= 0 || a.d <= 0 || a.traj_tokens < 0) return kWsHeader;
+  size_t b = kWsHeader + align256((size_t)a.hq * a.num_tokens * 4) + align256((size_t)a.num_tokens * a.hq * a.d * 4);
+  if (a.traj_tokens > 0)  // gathered: fp32 trajectory-layout dQ, dK, dV accumulators
+    b += align256((size_t)a.traj_tokens * a.hq * a.d * 4) + 2 * align256((size_t)a.traj_tokens * a.hkv * a.d * 4);
+  return b;
 }
 
 cudaError_t launch_attn_bwd(const AttnArgs& a, const void* o, const float* lse, const void* dout, void* dq, void* dk,
                             void* dv, void* ws, cudaStream_t st) {
-  if (a.d == 64) return launch_bwd_d<64>(a, o, lse, dout, dq, dk, dv, ws, st);
-  return launch_bwd_d<128>(a, o, lse, dout, dq, dk, dv, ws, st);
+  if (a.tok_gather != nullptr) {
+    if (a.d == 64) return launch_bwd_d<64, true>(a, o, lse, dout, dq, dk, dv, ws, st);
+    return launch_bwd_d<128, true>(a, o, lse, dout, dq, dk, dv, ws, st);
+  }
+  if (a.d == 64) return launch_bwd_d<64, false>(a, o, lse, dout, dq, dk, dv, ws, st);
+  return launch_bwd_d<128, false>(a, o, lse, dout, dq, dk, dv, ws, st);
 }
 
 }  // namespace vcs

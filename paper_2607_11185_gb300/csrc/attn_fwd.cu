@@ -114,13 +114,19 @@ __device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_tmem, uint6
     tc_mma_ts(tmem_d, p_tmem + kk * 8, desc_at(vd, kk * 16 * 128), C::IDESC_PV, kk > 0 ? 1u : acc0);
 }
 
-template <int D>
+// GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
+// tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr 3-D tiled
+// maps of the same tensors for tiles whose rows are one run of consecutive trajectory rows.
+// Otherwise tm_q/k/v are segment-layout tiled maps and tm_qr/kr/vr are unused.
+template <int D, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, const int32_t* __restrict__ cu_seqlens,
                     int32_t num_segments, int32_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv,
                     int32_t npairs, float scale_log2, __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
-                    int32_t* status) {
+                    int32_t* status, const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
+                    const __grid_constant__ CUtensorMap tm_qr, const __grid_constant__ CUtensorMap tm_kr,
+                    const __grid_constant__ CUtensorMap tm_vr) {
   using C = Fwd<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -181,35 +187,71 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp < 4) {
     setmaxnreg_dec<kRegCtrl>();
-    if (warp == 0 && lane == 0) {
+    if (warp == 0 && (GATHER || lane == 0)) {
     // ------------------------------------------------------------ producer
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      mbar_arrive_expect_tx(&bars->q_full, (has1 ? 2 : 1) * C::TILE);
-#pragma unroll
-      for (int kb = 0; kb < C::KB; ++kb) {
-        tma_load_3d(smem + C::OFF_Q0 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m0 * C::BM);
-        if (has1)
-          tma_load_3d(smem + C::OFF_Q1 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m1 * C::BM);
-      }
-      const uint64_t keep_l2 = l2_policy_evict_last();
-      // ring order K0, K1, V0, K2, V1, ..., K_{n-1}, V_{n-2}, V_{n-1}
-      for (int c = 0; c < 2 * nkv; ++c) {
-        const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
-        const int j = c == 2 * nkv - 1 ? nkv - 1 : (is_v ? (c - 2) >> 1 : (c + 1) >> 1);
-        const int slot = c % C::NSLOT, round = c / C::NSLOT;
-        if (c >= C::NSLOT && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
-          on_timeout(bars, status);
-          break;
+      if constexpr (GATHER) {
+        // the whole warp: lane 0 posts each tile's bytes and waits for free slots
+        if (lane == 0) {
+          tma_prefetch_desc(&tm_q);
+          tma_prefetch_desc(&tm_k);
+          tma_prefetch_desc(&tm_v);
+          mbar_arrive_expect_tx(&bars->q_full, (has1 ? 2 : 1) * C::TILE);
         }
-        if (aborted(bars)) break;
-        mbar_arrive_expect_tx(&bars->kv_full[slot], C::TILE);
-        const CUtensorMap* tm = is_v ? &tm_v : &tm_k;
+        __syncwarp();
+        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q0, &tm_q, &tm_qr, &bars->q_full, h, D, start + m0 * C::BM, end - 1,
+                                     tok_gather, traj_tokens, status, lane);
+        if (has1)
+          load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q1, &tm_q, &tm_qr, &bars->q_full, h, D, start + m1 * C::BM, end - 1,
+                                       tok_gather, traj_tokens, status, lane);
+        for (int c = 0; c < 2 * nkv; ++c) {
+          const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
+          const int j = c == 2 * nkv - 1 ? nkv - 1 : (is_v ? (c - 2) >> 1 : (c + 1) >> 1);
+          const int slot = c % C::NSLOT, round = c / C::NSLOT;
+          int go = 1;
+          if (lane == 0) {
+            if (c >= C::NSLOT && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
+              on_timeout(bars, status);
+              go = 0;
+            } else if (aborted(bars)) {
+              go = 0;
+            } else {
+              mbar_arrive_expect_tx(&bars->kv_full[slot], C::TILE);
+            }
+          }
+          if (!__shfl_sync(0xffffffffu, go, 0)) break;
+          load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_KV + slot * C::TILE, is_v ? &tm_v : &tm_k,
+                                          is_v ? &tm_vr : &tm_kr, &bars->kv_full[slot], g, D, start + j * C::BN,
+                                          end - 1, tok_gather, traj_tokens, status, lane);
+        }
+      } else {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_v);
+        mbar_arrive_expect_tx(&bars->q_full, (has1 ? 2 : 1) * C::TILE);
 #pragma unroll
-        for (int kb = 0; kb < C::KB; ++kb)
-          tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, &bars->kv_full[slot], kb * 64, g,
-                           start + j * C::BN, keep_l2);
+        for (int kb = 0; kb < C::KB; ++kb) {
+          tma_load_3d(smem + C::OFF_Q0 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m0 * C::BM);
+          if (has1)
+            tma_load_3d(smem + C::OFF_Q1 + kb * C::BLOCK, &tm_q, &bars->q_full, kb * 64, h, start + m1 * C::BM);
+        }
+        const uint64_t keep_l2 = l2_policy_evict_last();
+        // ring order K0, K1, V0, K2, V1, ..., K_{n-1}, V_{n-2}, V_{n-1}
+        for (int c = 0; c < 2 * nkv; ++c) {
+          const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
+          const int j = c == 2 * nkv - 1 ? nkv - 1 : (is_v ? (c - 2) >> 1 : (c + 1) >> 1);
+          const int slot = c % C::NSLOT, round = c / C::NSLOT;
+          if (c >= C::NSLOT && !mbar_wait(&bars->kv_empty[slot], (round - 1) & 1)) {
+            on_timeout(bars, status);
+            break;
+          }
+          if (aborted(bars)) break;
+          mbar_arrive_expect_tx(&bars->kv_full[slot], C::TILE);
+          const CUtensorMap* tm = is_v ? &tm_v : &tm_k;
+#pragma unroll
+          for (int kb = 0; kb < C::KB; ++kb)
+            tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, &bars->kv_full[slot], kb * 64, g,
+                             start + j * C::BN, keep_l2);
+        }
       }
     } else if (warp == 1 && lane == 0) {
     // ------------------------------------------------------------ MMA issuer
@@ -408,25 +450,34 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int D>
+template <int D, bool GATHER>
 cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st) {
   using C = Fwd<D>;
-  alignas(64) CUtensorMap tq, tk, tv;
-  if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
-      !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
-      !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128))
+  alignas(64) CUtensorMap tq, tk, tv, tqr, tkr, tvr;
+  if (GATHER) {
+    if (!encode_tma_rows_bf16(&tq, a.q, (uint64_t)a.hq * D, a.traj_tokens) ||
+        !encode_tma_rows_bf16(&tk, a.k, (uint64_t)a.hkv * D, a.traj_tokens) ||
+        !encode_tma_rows_bf16(&tv, a.v, (uint64_t)a.hkv * D, a.traj_tokens) ||
+        !encode_tma_3d_bf16(&tqr, a.q, D, a.hq, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tkr, a.k, D, a.hkv, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128))
+      return cudaErrorInvalidValue;
+  } else if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
+             !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
+             !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128)) {
     return cudaErrorInvalidValue;
+  }
   // the warpgroups' setmaxnreg targets are served from the registers the block
   // is launched with: refuse to launch a build that got a different count
   static int regs_ok = -1;
   if (regs_ok < 0) {
     cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, attn_fwd_kernel<D>);
+    cudaError_t e = cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, GATHER>);
     if (e != cudaSuccess) return e;
     regs_ok = fa.numRegs == kRegLaunch ? 1 : 0;
   }
   if (!regs_ok) return cudaErrorInvalidConfiguration;
-  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
   const int npairs = (a.max_seqlen + 2 * C::BM - 1) / (2 * C::BM);
   if (npairs == 0) return cudaSuccess;
@@ -434,9 +485,10 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
   if (gx > INT32_MAX) return cudaErrorInvalidConfiguration;
   const float scale_log2 = a.scale * 1.4426950408889634f;
   dim3 grid((unsigned)gx, 1, 1);
-  attn_fwd_kernel<D><<<grid, kThreads, C::SMEM, st>>>(tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens,
-                                                     a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
-                                                     static_cast<__nv_bfloat16*>(o), lse, a.status);
+  attn_fwd_kernel<D, GATHER><<<grid, kThreads, C::SMEM, st>>>(
+      tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
+      static_cast<__nv_bfloat16*>(o), lse, a.status, a.tok_gather, (int32_t)a.traj_tokens, GATHER ? tqr : tq,
+      GATHER ? tkr : tk, GATHER ? tvr : tv);
   return cudaGetLastError();
 }
 
@@ -449,8 +501,12 @@ size_t attn_fwd_ws_bytes(const AttnArgs& a) {
 
 cudaError_t launch_attn_fwd(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st) {
   (void)ws;
-  if (a.d == 64) return launch_fwd_d<64>(a, o, lse, st);
-  return launch_fwd_d<128>(a, o, lse, st);
+  if (a.tok_gather != nullptr) {
+    if (a.d == 64) return launch_fwd_d<64, true>(a, o, lse, st);
+    return launch_fwd_d<128, true>(a, o, lse, st);
+  }
+  if (a.d == 64) return launch_fwd_d<64, false>(a, o, lse, st);
+  return launch_fwd_d<128, false>(a, o, lse, st);
 }
 
 }  // namespace vcs

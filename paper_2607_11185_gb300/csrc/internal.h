@@ -53,6 +53,10 @@ struct AttnArgs {
   int32_t hq, hkv, d;
   float scale;
   int32_t* status;  // device status word (workspace header)
+  // gathered variants: q, k, v are trajectory-layout [traj_tokens, heads, d] tensors and
+  // segment token n reads trajectory row tok_gather[n]; nullptr for segment-layout inputs
+  const int32_t* tok_gather = nullptr;
+  int64_t traj_tokens = 0;
 };
 size_t attn_fwd_ws_bytes(const AttnArgs& a);
 cudaError_t launch_attn_fwd(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st);
@@ -83,6 +87,9 @@ bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d,
 
 // fp32 variant (bulk reduce-add targets): no swizzle, or the 128-byte swizzle
 // (box_d * 4 must then be 128).
+// 2-D map over a row-major [rows, row_elems] bf16 tensor with a 64-column x 1-row box and the
+// 128-byte swizzle: the map of the TMA gather4 loads (one row per gathered token)
+bool encode_tma_rows_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows);
 bool encode_tma_3d_f32(void* map, const void* base, uint64_t d, uint64_t heads, uint64_t tokens, uint32_t box_d,
                        uint32_t box_rows, bool swizzle128 = false);
 

@@ -293,5 +293,58 @@ __device__ __forceinline__ void set_status(int32_t* status, int32_t code) {
   if (status != nullptr) atomicCAS(status, 0, code);
 }
 
+// ---------------------------------------------------------------- gathered tiles
+// TMA gather4: four rows r0..r3 (the outer coordinate of a 2-D tensor map whose box is
+// 64 columns x 1 row) from column col, written as four consecutive 128-byte rows at dst.
+// The 128-byte swizzle is applied by shared-memory address, so rows gathered to
+// dst = tile + 128 * i land exactly where a tiled load of the same rows would put them.
+__device__ __forceinline__ void tma_gather4(void* dst, const void* map, uint64_t* bar, int col, int r0, int r1, int r2,
+                                            int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, "
+      "%5, %6, %7}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(smem_u32(bar)), "r"(col), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
+      : "memory");
+}
+
+// One warp loads the 128-row tile of segment rows s0 .. s0+127 (rows past `last` repeat
+// row `last`) of one head from a trajectory-layout tensor through the gather map.  When the
+// tile's 128 rows are consecutive trajectory rows (inside a screenshot-and-text run of the
+// segment) lane 0 issues the KB tiled loads of the 3-D map tmap (box 64 x 1 head x 128 rows);
+// otherwise lane l gathers rows 4l .. 4l+3 of each 64-column block with the 2-D map gmap, to
+// the same swizzled positions.  Blocks are BLOCK bytes apart at dst.  A gather index outside
+// [0, traj_tokens) is recorded as a device check and read as row 0.  The caller has posted
+// the tile's bytes on `bar`.
+template <int KB, int BLOCK>
+__device__ __forceinline__ void load_traj_tile(uint8_t* dst, const void* gmap, const void* tmap, uint64_t* bar,
+                                               int head, int d, int s0, int last,
+                                               const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
+                                               int32_t* status, int lane) {
+  int t[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = min(s0 + 4 * lane + i, last);
+    t[i] = __ldg(&tok_gather[row]);
+    if (t[i] < 0 || t[i] >= traj_tokens) {
+      set_status(status, 6 /* VCS_ERR_DEVICE_CHECK */);
+      t[i] = 0;
+    }
+  }
+  const int base = __shfl_sync(0xffffffffu, t[0], 0);
+  bool run = s0 + 127 <= last;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) run = run && t[i] == base + 4 * lane + i;
+  if (__all_sync(0xffffffffu, run)) {
+    if (lane == 0) {
+#pragma unroll
+      for (int kb = 0; kb < KB; ++kb) tma_load_3d(dst + kb * BLOCK, tmap, bar, kb * 64, head, base);
+    }
+  } else {
+#pragma unroll
+    for (int kb = 0; kb < KB; ++kb)
+      tma_gather4(dst + kb * BLOCK + lane * 512, gmap, bar, head * d + kb * 64, t[0], t[1], t[2], t[3]);
+  }
+}
+
 }  // namespace dev
 }  // namespace vcs

@@ -59,6 +59,12 @@ _lib_bwd = _sig("vcs_attn_bwd", _i32,
 
 _lib_bwd_noalloc = _sig("vcs_attn_bwd_noalloc", _i32,
                         [_p, _p, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p, _p])
+_lib_fwd_g = _sig("vcs_attn_fwd_gathered", _i32,
+                  [_p, _p, _p, _i64, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _sz, _p])
+_lib_bwd_g_ws = _sig("vcs_attn_bwd_gathered_workspace_size", _sz, [_i32, _i64, _i32, _i64, _i32, _i32, _i32])
+_lib_bwd_g = _sig("vcs_attn_bwd_gathered", _i32,
+                  [_p, _p, _p, _i64, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p,
+                   _sz, _p])
 
 _f64 = ctypes.c_double
 _lib_loss_ws = _sig("vcs_grpo_loss_workspace_size", _sz, [_i64])
@@ -73,7 +79,8 @@ EXPORTED = ["vcs_status_string", "vcs_version", "vcs_segments_workspace_size", "
             "vcs_build_segments", "vcs_gather", "vcs_attn_fwd_workspace_size", "vcs_attn_fwd",
             "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc", "vcs_grpo_loss_workspace_size",
             "vcs_grpo_loss", "vcs_group_advantage", "vcs_stream_fields", "vcs_compact_workspace_size",
-            "vcs_compact_trainable"]
+            "vcs_compact_trainable", "vcs_attn_fwd_gathered", "vcs_attn_bwd_gathered_workspace_size",
+            "vcs_attn_bwd_gathered"]
 
 LIB_PATH = _LIB_PATH
 
@@ -156,6 +163,25 @@ def vcs_attn_bwd(q, k, v, o, lse, dout, cu_seqlens, num_segments, num_tokens, ma
     return _lib_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout), _ptr(cu_seqlens), num_segments,
                     num_tokens, max_seqlen, hq, hkv, d, softmax_scale, _ptr(dq), _ptr(dk), _ptr(dv), _ptr(ws),
                     ws_bytes, _stream(stream))
+
+
+def vcs_attn_fwd_gathered(q_traj, k_traj, v_traj, traj_tokens, tok_gather, cu_seqlens, num_segments, num_tokens,
+                          max_seqlen, hq, hkv, d, softmax_scale, o, lse, ws, ws_bytes, stream=None) -> int:
+    return _lib_fwd_g(_ptr(q_traj), _ptr(k_traj), _ptr(v_traj), traj_tokens, _ptr(tok_gather), _ptr(cu_seqlens),
+                      num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale, _ptr(o), _ptr(lse), _ptr(ws),
+                      ws_bytes, _stream(stream))
+
+
+def vcs_attn_bwd_gathered_workspace_size(num_segments, num_tokens, max_seqlen, traj_tokens, hq, hkv, d) -> int:
+    return int(_lib_bwd_g_ws(num_segments, num_tokens, max_seqlen, traj_tokens, hq, hkv, d))
+
+
+def vcs_attn_bwd_gathered(q_traj, k_traj, v_traj, traj_tokens, tok_gather, o, lse, dout, cu_seqlens, num_segments,
+                          num_tokens, max_seqlen, hq, hkv, d, softmax_scale, dq_traj, dk_traj, dv_traj, ws, ws_bytes,
+                          stream=None) -> int:
+    return _lib_bwd_g(_ptr(q_traj), _ptr(k_traj), _ptr(v_traj), traj_tokens, _ptr(tok_gather), _ptr(o), _ptr(lse),
+                      _ptr(dout), _ptr(cu_seqlens), num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale,
+                      _ptr(dq_traj), _ptr(dk_traj), _ptr(dv_traj), _ptr(ws), ws_bytes, _stream(stream))
 
 
 def vcs_attn_bwd_noalloc(q, k, v, o, lse, dout, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d,
@@ -298,6 +324,44 @@ def attn_bwd(q, k, v, o, lse, dout, cu_seqlens, max_seqlen: int, softmax_scale: 
                         dv, ws, nb, stream), "vcs_attn_bwd")
     if check:
         _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_bwd (device)")
+    return dq, dk, dv
+
+
+def attn_fwd_gathered(q_traj, k_traj, v_traj, tok_gather, cu_seqlens, max_seqlen: int, softmax_scale: float = 0.0,
+                      stream=None, check=True):
+    """Attention forward over the segments, reading trajectory-layout q/k/v through tok_gather;
+    o [num_tokens, hq, d] and lse [hq, num_tokens] in segment layout."""
+    tt, hq, d = q_traj.shape
+    hkv = k_traj.shape[1]
+    nt = tok_gather.numel()
+    ns = cu_seqlens.numel() - 1
+    o = torch.empty((nt, hq, d), dtype=q_traj.dtype, device=q_traj.device)
+    lse = torch.empty((hq, nt), dtype=torch.float32, device=q_traj.device)
+    nb = vcs_attn_fwd_workspace_size(ns, nt, max_seqlen, hq, hkv, d)
+    ws = _ws(nb, q_traj.device)
+    _check(vcs_attn_fwd_gathered(q_traj, k_traj, v_traj, tt, tok_gather, cu_seqlens, ns, nt, max_seqlen, hq, hkv, d,
+                                 softmax_scale, o, lse, ws, nb, stream), "vcs_attn_fwd_gathered")
+    if check:
+        _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_fwd_gathered (device)")
+    return o, lse
+
+
+def attn_bwd_gathered(q_traj, k_traj, v_traj, tok_gather, o, lse, dout, cu_seqlens, max_seqlen: int,
+                      softmax_scale: float = 0.0, stream=None, check=True):
+    """Attention backward over the segments with trajectory-layout q/k/v read through tok_gather;
+    returns dq, dk, dv in trajectory layout (each token's segment copies summed)."""
+    tt, hq, d = q_traj.shape
+    hkv = k_traj.shape[1]
+    nt = tok_gather.numel()
+    ns = cu_seqlens.numel() - 1
+    dq, dk, dv = torch.empty_like(q_traj), torch.empty_like(k_traj), torch.empty_like(v_traj)
+    nb = vcs_attn_bwd_gathered_workspace_size(ns, nt, max_seqlen, tt, hq, hkv, d)
+    ws = _ws(nb, q_traj.device)
+    _check(vcs_attn_bwd_gathered(q_traj, k_traj, v_traj, tt, tok_gather, o, lse, dout, cu_seqlens, ns, nt,
+                                 max_seqlen, hq, hkv, d, softmax_scale, dq, dk, dv, ws, nb, stream),
+           "vcs_attn_bwd_gathered")
+    if check:
+        _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_bwd_gathered (device)")
     return dq, dk, dv
 
 
