@@ -328,6 +328,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next-rows", action="store_true", help="skip the stream-field / loss kernel timings")
     ap.add_argument("--no-fused", action="store_true", help="skip the gathered-attention (fused gather) timing")
+    ap.add_argument("--no-reuse", action="store_true", help="skip the prefix-reuse forward timing")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -406,6 +407,7 @@ def main():
 
     next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
     fused = None if args.no_fused else run_fused(path, stream)
+    reuse = None if args.no_reuse else run_reuse(path, stream)
 
     ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
     line = {
@@ -433,6 +435,7 @@ def main():
         "e2e": e2e,
         "next_rows": next_rows,
         "fused_gather": fused,
+        "prefix_reuse": reuse,
         "gpu_launches": path.launches_per_step * args.steps,
         "clocks": ck,
     }
@@ -561,6 +564,60 @@ def run_fused(path, stream, reps=2):
                             "(fp32 sums over each token's copies)")
     out["materialised"]["note"] = "gather + forward + backward, gradients left in segment layout"
     del gws, dqt, dkt, dvt
+    return out
+
+
+def run_reuse(path, stream, reps=3):
+    """Forward with prefix reuse (each query-tile pair whose rows a trajectory's previous
+    segment shares is copied, not computed) against the plain forward, on the largest
+    chunk: vcs_shared_prefix, vcs_attn_fwd_reuse and vcs_attn_fwd timed with CUDA events,
+    1 warm-up + `reps` timed launches each.  TFLOP/s are the plain forward's credited flops
+    over each time, so the ratio is the speed-up."""
+    vcs, w = path.vcs, path.w
+    hq, hkv, d = w.hq, w.hkv, w.d
+    ci = path.chunk_in[0]
+    sp = stream.cuda_stream
+    nseg, ntok, mx = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"], ci["max_seqlen"]
+    seg_traj = torch.empty(path.max_seg, dtype=torch.int32, device=path.dev)
+    assert vcs.vcs_build_segments(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"], path.window,
+                                  path.keep, path.max_seg, path.max_tok, path.cu_seqlens, seg_traj, path.tok_gather,
+                                  path.tok_src, path.tok_pos, path.tok_mask, path.sizes, path.seg_ws,
+                                  path.seg_ws_bytes, sp) == 0
+    qt, kt, vt = (x[ci["ttok0"]:ci["ttok1"]] for x in (path.q_traj, path.k_traj, path.v_traj))
+    assert vcs.vcs_gather(qt, kt, vt, ci["ttok1"] - ci["ttok0"], path.tok_gather, ntok, hq, hkv, d, path.q, path.k,
+                          path.v, path.gstatus, sp) == 0
+    shared = torch.empty(nseg, dtype=torch.int32, device=path.dev)
+    status = torch.zeros(1, dtype=torch.int32, device=path.dev)
+    calls = {
+        "shared_prefix_ms": lambda: vcs.vcs_shared_prefix(path.cu_seqlens, seg_traj, path.tok_gather, nseg, ntok,
+                                                          shared, status, sp),
+        "fwd_reuse_ms": lambda: vcs.vcs_attn_fwd_reuse(path.q, path.k, path.v, path.cu_seqlens, shared, nseg, ntok, mx,
+                                                       hq, hkv, d, 0.0, path.o, path.lse, path.fwd_ws,
+                                                       path.fwd_ws_bytes, sp),
+        "fwd_ms": lambda: vcs.vcs_attn_fwd(path.q, path.k, path.v, path.cu_seqlens, nseg, ntok, mx, hq, hkv, d, 0.0,
+                                           path.o, path.lse, path.fwd_ws, path.fwd_ws_bytes, sp),
+    }
+    out = {"chunk_segment_tokens": ntok}
+    for name, fn in calls.items():
+        times = []
+        for i in range(1 + reps):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            e[0].record(stream)
+            assert fn() == 0, name
+            e[1].record(stream)
+            if i > 0:
+                times.append(e)
+        torch.cuda.synchronize()
+        out[name] = statistics.mean(a.elapsed_time(b) for a, b in times)
+    assert int(status.item()) == 0 and path.device_status() == (0, 0, 0)
+    # credited forward flops of the skipped pairs (their rows are copied) against the chunk's
+    lens = path.seg_lens[ci["s0"]:ci["s1"]].astype(np.int64)
+    skip = shared.cpu().numpy().astype(np.int64) // 256 * 256
+    _, f_all, _ = credited_flops(lens, hq, d)
+    _, f_skip, _ = credited_flops(skip, hq, d)
+    out["skipped_flop_frac"] = f_skip / f_all
+    out["fwd_tflops"] = f_all / (out["fwd_ms"] / 1e3) / 1e12
+    out["fwd_reuse_tflops_equiv"] = f_all / (out["fwd_reuse_ms"] / 1e3) / 1e12
     return out
 
 

@@ -257,6 +257,43 @@ vcs_status vcs_attn_bwd_gathered(const void* q_traj, const void* k_traj, const v
                                  void* stream);
 
 /* ------------------------------------------------------------------------
+ * Prefix reuse (forward).  A fresh stream re-tokenises the text of the steps
+ * before its window (Alg. 1, Sec. 3.4 / App. C.1) and the steps that leave the
+ * window join that text, so a trajectory's segment s starts with the tokens
+ * its segment s-1 starts with.  Causal attention row r depends only on tokens
+ * 0..r of its segment (positions restart at 0 in every stream), so over the
+ * common prefix the two segments' rows are equal.  The paper does not use
+ * this; it only removes repeated forward work.
+ *
+ * vcs_shared_prefix: seg_shared[s] = the largest n <= min(L_s, L_{s-1}) with
+ * tok_gather[cu[s] + i] == tok_gather[cu[s-1] + i] for all i < n, and 0 when
+ * seg_traj[s] != seg_traj[s-1] or s = 0.
+ *   cu_seqlens, seg_traj, tok_gather  from vcs_build_segments (device)
+ *   seg_shared  int32 [num_segments] device (written)
+ *   dev_status  int32 device word or NULL: VCS_ERR_DEVICE_CHECK for
+ *               inconsistent cu_seqlens (that segment gets 0)
+ *
+ * vcs_attn_fwd_reuse: vcs_attn_fwd's result (bit for bit) with seg_shared
+ * from vcs_shared_prefix: the query-tile pairs (256 rows) of segment s that
+ * lie wholly below seg_shared[s] are not computed; their o and lse rows are
+ * copied from the segment that computed them (going back through the
+ * trajectory's segments).  Arguments and errors as vcs_attn_fwd, plus
+ * VCS_ERR_INVALID_ARG for a NULL seg_shared with segments present; a
+ * seg_shared[s] larger than either segment, negative, or non-zero for s = 0
+ * is recorded as VCS_ERR_DEVICE_CHECK in the workspace status word and read
+ * as 0.  (A seg_shared larger than the true common prefix gives wrong rows,
+ * not a fault: pass vcs_shared_prefix's.)
+ * ------------------------------------------------------------------------ */
+vcs_status vcs_shared_prefix(const int32_t* cu_seqlens, const int32_t* seg_traj, const int32_t* tok_gather,
+                             int32_t num_segments, int64_t num_tokens, int32_t* seg_shared, int32_t* dev_status,
+                             void* stream);
+
+vcs_status vcs_attn_fwd_reuse(const void* q, const void* k, const void* v, const int32_t* cu_seqlens,
+                              const int32_t* seg_shared, int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                              int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* o, float* lse, void* ws,
+                              size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * Token-ID stream fields (App. C.1, Algorithm 1's (ids, mask, logp) stream).
  * Response tokens enter a segment's stream as trainable tokens with their
  * rollout log-probabilities; observation tokens and the re-tokenised history

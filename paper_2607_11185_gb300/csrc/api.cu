@@ -325,6 +325,42 @@ vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void*
   return VCS_OK;
 }
 
+// ---------------------------------------------------------------- prefix reuse
+vcs_status vcs_shared_prefix(const int32_t* cu_seqlens, const int32_t* seg_traj, const int32_t* tok_gather,
+                             int32_t num_segments, int64_t num_tokens, int32_t* seg_shared, int32_t* dev_status,
+                             void* stream) {
+  if (num_segments < 0 || num_tokens < 0) return VCS_ERR_INVALID_ARG;
+  if (num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
+  if (num_segments > 0 && (cu_seqlens == nullptr || seg_traj == nullptr || seg_shared == nullptr ||
+                           (num_tokens > 0 && tok_gather == nullptr)))
+    return VCS_ERR_INVALID_ARG;
+  if (launch_shared_prefix(cu_seqlens, seg_traj, tok_gather, num_segments, (int32_t)num_tokens, seg_shared,
+                           dev_status, as_stream(stream)) != cudaSuccess)
+    return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
+vcs_status vcs_attn_fwd_reuse(const void* q, const void* k, const void* v, const int32_t* cu_seqlens,
+                              const int32_t* seg_shared, int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
+                              int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* o, float* lse, void* ws,
+                              size_t ws_bytes, void* stream) {
+  AttnArgs a = make_args(q, k, v, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
+  vcs_status s = check_attn(a);
+  if (s != VCS_OK) return s;
+  if (num_segments > 0 && seg_shared == nullptr) return VCS_ERR_INVALID_ARG;
+  a.seg_shared = seg_shared;
+  if ((num_tokens > 0 && (o == nullptr || lse == nullptr)) || !aligned16(o) || !aligned16(lse))
+    return VCS_ERR_INVALID_ARG;
+  if (ws == nullptr || ws_bytes < attn_fwd_ws_bytes(a) || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0)
+    return VCS_ERR_WORKSPACE;
+  a.status = static_cast<int32_t*>(ws);
+  cudaStream_t st = as_stream(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, st) != cudaSuccess) return VCS_ERR_CUDA;
+  if (num_tokens == 0 || num_segments == 0) return VCS_OK;
+  if (launch_attn_fwd(a, o, lse, ws, st) != cudaSuccess) return VCS_ERR_CUDA;
+  return VCS_OK;
+}
+
 // ---------------------------------------------------------------- gathered attention
 // The attention forward/backward reading Q, K, V straight from trajectory-layout tensors
 // through the builder's gather map (no materialised segment-layout copies); the backward

@@ -114,6 +114,24 @@ __device__ __forceinline__ void issue_pv(uint32_t tmem_d, uint32_t p_tmem, uint6
     tc_mma_ts(tmem_d, p_tmem + kk * 8, desc_at(vd, kk * 16 * 128), C::IDESC_PV, kk > 0 ? 1u : acc0);
 }
 
+// Prefix reuse: rows [0, skip) of segment s, skip the shared prefix with segment s-1
+// rounded down to whole pairs of query tiles, equal rows [0, skip) of segment s-1 and are
+// copied from there instead of computed.  A shared length that segment s-1 cannot have
+// (negative, longer than either segment, or given for segment 0) is recorded as a device
+// check and read as 0.
+__device__ __forceinline__ int reuse_skip_rows(const int32_t* __restrict__ seg_shared,
+                                               const int32_t* __restrict__ cu_seqlens, int s, int32_t* status) {
+  if (seg_shared == nullptr) return 0;
+  const int sh = seg_shared[s];
+  if (sh == 0) return 0;
+  const int L = cu_seqlens[s + 1] - cu_seqlens[s];
+  if (s == 0 || sh < 0 || sh > L || sh > cu_seqlens[s] - cu_seqlens[s - 1]) {
+    set_status(status, VCS_ERR_DEVICE_CHECK);
+    return 0;
+  }
+  return sh / 256 * 256;
+}
+
 // GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
 // tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr 3-D tiled
 // maps of the same tensors for tiles whose rows are one run of consecutive trajectory rows.
@@ -126,7 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     int32_t npairs, float scale_log2, __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
                     int32_t* status, const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
                     const __grid_constant__ CUtensorMap tm_qr, const __grid_constant__ CUtensorMap tm_kr,
-                    const __grid_constant__ CUtensorMap tm_vr) {
+                    const __grid_constant__ CUtensorMap tm_vr, const int32_t* __restrict__ seg_shared) {
   using C = Fwd<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -155,6 +173,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   const int L = end - start;
   if (p * 2 * C::BM >= L) return;  // this pair of query tiles lies beyond the segment
+  // prefix reuse: the pair's rows equal the previous segment's (copied by fwd_reuse_copy)
+  if (seg_shared != nullptr && (p + 1) * 2 * C::BM <= reuse_skip_rows(seg_shared, cu_seqlens, seg, status)) return;
   const int m0 = 2 * p, m1 = 2 * p + 1;
   const bool has1 = m1 * C::BM < L;
   const int nkv = has1 ? m1 + 1 : m0 + 1;
@@ -450,6 +470,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Prefix reuse: O and lse of the rows the forward skipped, from the segment that computed
+// them (walk back through the previous segments while the row lies in their skipped
+// prefix).  One warp per segment token; 16-byte pieces of the O row, then the lse values.
+__global__ void __launch_bounds__(256) fwd_reuse_copy(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
+                                                      int32_t num_tokens, const int32_t* __restrict__ seg_shared,
+                                                      int32_t hq, int32_t d, __nv_bfloat16* __restrict__ out,
+                                                      float* __restrict__ lse, int32_t* status) {
+  const int warps = gridDim.x * 8;
+  const int lane = threadIdx.x & 31;
+  for (int n = blockIdx.x * 8 + (threadIdx.x >> 5); n < num_tokens; n += warps) {
+    int lo = 0, hi = num_segments - 1;  // the segment s with cu[s] <= n < cu[s+1]
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (cu_seqlens[mid] <= n) lo = mid;
+      else hi = mid - 1;
+    }
+    const int r = n - cu_seqlens[lo];
+    int src = lo;
+    while (r < reuse_skip_rows(seg_shared, cu_seqlens, src, status)) --src;
+    if (src == lo) continue;
+    const int m = cu_seqlens[src] + r;  // the same row of the segment that computed it
+    const int chunks = hq * d / 8;
+    const uint4* from = reinterpret_cast<const uint4*>(out + (size_t)m * hq * d);
+    uint4* to = reinterpret_cast<uint4*>(out + (size_t)n * hq * d);
+    for (int c = lane; c < chunks; c += 32) to[c] = from[c];
+    for (int h = lane; h < hq; h += 32) lse[(size_t)h * num_tokens + n] = lse[(size_t)h * num_tokens + m];
+  }
+}
+
 template <int D, bool GATHER>
 cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st) {
   using C = Fwd<D>;
@@ -488,7 +537,16 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
   attn_fwd_kernel<D, GATHER><<<grid, kThreads, C::SMEM, st>>>(
       tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
       static_cast<__nv_bfloat16*>(o), lse, a.status, a.tok_gather, (int32_t)a.traj_tokens, GATHER ? tqr : tq,
-      GATHER ? tkr : tk, GATHER ? tvr : tv);
+      GATHER ? tkr : tk, GATHER ? tvr : tv, a.seg_shared);
+  if (a.seg_shared != nullptr) {
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    int64_t blocks = (a.num_tokens + 7) / 8;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    fwd_reuse_copy<<<(unsigned)blocks, 256, 0, st>>>(a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens,
+                                                     a.seg_shared, a.hq, D, static_cast<__nv_bfloat16*>(o), lse,
+                                                     a.status);
+  }
   return cudaGetLastError();
 }
 

@@ -57,6 +57,9 @@ struct AttnArgs {
   // segment token n reads trajectory row tok_gather[n]; nullptr for segment-layout inputs
   const int32_t* tok_gather = nullptr;
   int64_t traj_tokens = 0;
+  // prefix reuse (forward): per segment, the length of its common prefix with the previous
+  // segment of its trajectory (vcs_shared_prefix); nullptr computes every row
+  const int32_t* seg_shared = nullptr;
 };
 size_t attn_fwd_ws_bytes(const AttnArgs& a);
 cudaError_t launch_attn_fwd(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st);
@@ -80,6 +83,10 @@ cudaError_t launch_stream_fields(const int32_t* traj_ids, const float* traj_logp
 size_t compact_ws_bytes(int64_t num_tokens);
 cudaError_t launch_compact(const uint8_t* mask, int64_t num_tokens, int32_t* idx, int64_t capacity, int64_t* count,
                            void* ws, cudaStream_t st);
+
+cudaError_t launch_shared_prefix(const int32_t* cu_seqlens, const int32_t* seg_traj, const int32_t* tok_gather,
+                                 int32_t num_segments, int32_t num_tokens, int32_t* seg_shared, int32_t* status,
+                                 cudaStream_t st);
 
 // TMA descriptor encoding through the driver entry point (no libcuda link).
 bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d, uint64_t heads, uint64_t tokens,

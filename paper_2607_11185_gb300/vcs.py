@@ -61,6 +61,9 @@ _lib_bwd_noalloc = _sig("vcs_attn_bwd_noalloc", _i32,
                         [_p, _p, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p, _p])
 _lib_fwd_g = _sig("vcs_attn_fwd_gathered", _i32,
                   [_p, _p, _p, _i64, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _sz, _p])
+_lib_shared = _sig("vcs_shared_prefix", _i32, [_p, _p, _p, _i32, _i64, _p, _p, _p])
+_lib_fwd_reuse = _sig("vcs_attn_fwd_reuse", _i32,
+                      [_p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _sz, _p])
 _lib_bwd_g_ws = _sig("vcs_attn_bwd_gathered_workspace_size", _sz, [_i32, _i64, _i32, _i64, _i32, _i32, _i32])
 _lib_bwd_g = _sig("vcs_attn_bwd_gathered", _i32,
                   [_p, _p, _p, _i64, _p, _p, _p, _p, _p, _i32, _i64, _i32, _i32, _i32, _i32, _f32, _p, _p, _p, _p,
@@ -80,7 +83,7 @@ EXPORTED = ["vcs_status_string", "vcs_version", "vcs_segments_workspace_size", "
             "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc", "vcs_grpo_loss_workspace_size",
             "vcs_grpo_loss", "vcs_group_advantage", "vcs_stream_fields", "vcs_compact_workspace_size",
             "vcs_compact_trainable", "vcs_attn_fwd_gathered", "vcs_attn_bwd_gathered_workspace_size",
-            "vcs_attn_bwd_gathered"]
+            "vcs_attn_bwd_gathered", "vcs_shared_prefix", "vcs_attn_fwd_reuse"]
 
 LIB_PATH = _LIB_PATH
 
@@ -170,6 +173,19 @@ def vcs_attn_fwd_gathered(q_traj, k_traj, v_traj, traj_tokens, tok_gather, cu_se
     return _lib_fwd_g(_ptr(q_traj), _ptr(k_traj), _ptr(v_traj), traj_tokens, _ptr(tok_gather), _ptr(cu_seqlens),
                       num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale, _ptr(o), _ptr(lse), _ptr(ws),
                       ws_bytes, _stream(stream))
+
+
+def vcs_shared_prefix(cu_seqlens, seg_traj, tok_gather, num_segments, num_tokens, seg_shared, dev_status=None,
+                      stream=None) -> int:
+    return _lib_shared(_ptr(cu_seqlens), _ptr(seg_traj), _ptr(tok_gather), num_segments, num_tokens,
+                       _ptr(seg_shared), _ptr(dev_status), _stream(stream))
+
+
+def vcs_attn_fwd_reuse(q, k, v, cu_seqlens, seg_shared, num_segments, num_tokens, max_seqlen, hq, hkv, d,
+                       softmax_scale, o, lse, ws, ws_bytes, stream=None) -> int:
+    return _lib_fwd_reuse(_ptr(q), _ptr(k), _ptr(v), _ptr(cu_seqlens), _ptr(seg_shared), num_segments, num_tokens,
+                          max_seqlen, hq, hkv, d, softmax_scale, _ptr(o), _ptr(lse), _ptr(ws), ws_bytes,
+                          _stream(stream))
 
 
 def vcs_attn_bwd_gathered_workspace_size(num_segments, num_tokens, max_seqlen, traj_tokens, hq, hkv, d) -> int:
@@ -325,6 +341,34 @@ def attn_bwd(q, k, v, o, lse, dout, cu_seqlens, max_seqlen: int, softmax_scale: 
     if check:
         _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_bwd (device)")
     return dq, dk, dv
+
+
+def shared_prefix(cu_seqlens, seg_traj, tok_gather, stream=None):
+    """Per segment, its common prefix length with the previous segment of its trajectory."""
+    ns = cu_seqlens.numel() - 1
+    out = torch.empty(max(ns, 0), dtype=torch.int32, device=cu_seqlens.device)
+    status = torch.zeros(1, dtype=torch.int32, device=cu_seqlens.device)
+    _check(vcs_shared_prefix(cu_seqlens, seg_traj, tok_gather, ns, tok_gather.numel(), out, status, stream),
+           "vcs_shared_prefix")
+    _check(int(status.item()), "vcs_shared_prefix (device)")
+    return out
+
+
+def attn_fwd_reuse(q, k, v, cu_seqlens, seg_shared, max_seqlen: int, softmax_scale: float = 0.0, stream=None,
+                   check=True):
+    """vcs_attn_fwd's o and lse, computing each shared prefix row once per trajectory."""
+    nt, hq, d = q.shape
+    hkv = k.shape[1]
+    ns = cu_seqlens.numel() - 1
+    o = torch.empty_like(q)
+    lse = torch.empty((hq, nt), dtype=torch.float32, device=q.device)
+    nb = vcs_attn_fwd_workspace_size(ns, nt, max_seqlen, hq, hkv, d)
+    ws = _ws(nb, q.device)
+    _check(vcs_attn_fwd_reuse(q, k, v, cu_seqlens, seg_shared, ns, nt, max_seqlen, hq, hkv, d, softmax_scale, o, lse,
+                              ws, nb, stream), "vcs_attn_fwd_reuse")
+    if check:
+        _check(int(ws[:4].view(torch.int32).item()), "vcs_attn_fwd_reuse (device)")
+    return o, lse
 
 
 def attn_fwd_gathered(q_traj, k_traj, v_traj, tok_gather, cu_seqlens, max_seqlen: int, softmax_scale: float = 0.0,
