@@ -302,10 +302,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_commit(&bars->kv_empty[0]);
       }
+      // V_0 and K_1 for the first step; every later step's V and K are acquired one step
+      // ahead, between the two tiles' issues, while the tensor pipe still has queued work
+      // (a barrier wait costs hundreds of cycles while the pipe streams from shared memory)
+      uint32_t vaddr_next = 0, kaddr_next = 0;
+      if (ok) ok = acquire(v_item(0), vaddr);
+      if (ok && nkv > 1) ok = acquire(k_item(1), kaddr);
       for (int j = 0; ok && j < nkv; ++j) {
         const bool next = j + 1 < nkv;
-        if (!acquire(v_item(j), vaddr)) { ok = false; break; }
-        if (next && !acquire(k_item(j + 1), kaddr)) { ok = false; break; }
         // tile 0: O0 += P0(j) V_j, then S0(j+1)
         if (j <= m0) {
           if (!mbar_wait(&bars->p_full[0], j & 1)) { ok = false; break; }
@@ -318,6 +322,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_commit(&bars->o_done[0]);
           }
         }
+        if (next && !acquire(v_item(j + 1), vaddr_next)) { ok = false; break; }
+        if (j + 2 < nkv && !acquire(k_item(j + 2), kaddr_next)) { ok = false; break; }
         // tile 1
         if (has1) {
           if (!mbar_wait(&bars->p_full[1], j & 1)) { ok = false; break; }
@@ -332,7 +338,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (next) tc_commit(&bars->kv_empty[k_item(j + 1) % C::NSLOT]);
         tc_commit(&bars->kv_empty[v_item(j) % C::NSLOT]);
-        if (aborted(bars)) { ok = false; break; }
+        vaddr = vaddr_next;
+        kaddr = kaddr_next;
       }
       if (!ok) on_timeout(bars, status);
     }
