@@ -1043,14 +1043,15 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   float* dvec = reinterpret_cast<float*>(w);
   float* dq_acc = reinterpret_cast<float*>(w + align256((size_t)a.hq * a.num_tokens * 4));
   // gathered: fp32 trajectory-layout accumulators of dQ, dK, dV after the segment-layout dQ
-  float* dq_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dq_acc) + align256((size_t)a.num_tokens * a.hq * D * 4));
-  float* dk_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dq_t) + align256((size_t)a.traj_tokens * a.hq * D * 4));
-  float* dv_t = reinterpret_cast<float*>(reinterpret_cast<char*>(dk_t) + align256((size_t)a.traj_tokens * a.hkv * D * 4));
+  float *dq_t = nullptr, *dk_t = nullptr, *dv_t = nullptr;
   const int64_t rows = a.num_tokens * a.hq;
   if (GATHER) {
-    const size_t span = reinterpret_cast<char*>(dv_t) - reinterpret_cast<char*>(dq_t) +
-                        (size_t)a.traj_tokens * a.hkv * D * 4;  // dq_t .. end of dv_t
-    if (cudaMemsetAsync(dq_t, 0, span, st) != cudaSuccess) return cudaErrorUnknown;
+    char* t0 = reinterpret_cast<char*>(dq_acc) + align256((size_t)a.num_tokens * a.hq * D * 4);
+    const size_t qb = align256((size_t)a.traj_tokens * a.hq * D * 4), kb = align256((size_t)a.traj_tokens * a.hkv * D * 4);
+    dq_t = reinterpret_cast<float*>(t0);
+    dk_t = reinterpret_cast<float*>(t0 + qb);
+    dv_t = reinterpret_cast<float*>(t0 + qb + kb);
+    if (cudaMemsetAsync(t0, 0, qb + 2 * kb, st) != cudaSuccess) return cudaErrorUnknown;
   }
   {
     const int64_t total = rows * (D / 8);

@@ -59,3 +59,41 @@ def test_host_side_argument_errors_without_gpu(lib):
     lib.vcs_attn_fwd_workspace_size.restype = ctypes.c_size_t
     lib.vcs_attn_fwd_workspace_size.argtypes = [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 4
     assert g(256, 256, 256, 256, 1, 10, 10, 2, 1, 64, 0.0, 256, 256, 256, 0, None) == 8      # no workspace
+
+
+def test_gathered_and_reuse_host_checks_without_gpu(lib):
+    # size queries are host arithmetic; argument errors return before any CUDA call
+    ws = lib.vcs_attn_bwd_workspace_size
+    ws.restype = ctypes.c_size_t
+    ws.argtypes = [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 4
+    gws = lib.vcs_attn_bwd_gathered_workspace_size
+    gws.restype = ctypes.c_size_t
+    gws.argtypes = [ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 3
+    r256 = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    for nt, tt, hq, hkv, d in ((1000, 700, 28, 4, 128), (17, 5, 2, 1, 64)):
+        assert gws(3, nt, 500, tt, hq, hkv, d) == ws(3, nt, 500, hq, hkv, d) + r256(tt * hq * d * 4) + 2 * r256(
+            tt * hkv * d * 4)
+        assert gws(3, nt, 500, 0, hq, hkv, d) == ws(3, nt, 500, hq, hkv, d)
+    f = lib.vcs_attn_fwd_gathered
+    f.restype = ctypes.c_int32
+    f.argtypes = [ctypes.c_void_p] * 3 + [ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int32,
+                                          ctypes.c_int64] + [ctypes.c_int32] * 4 + [ctypes.c_float] + \
+        [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p]
+    A = 256
+    assert f(A, A, A, 100, None, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 4096, None) == 1        # no gather map
+    assert f(A, A, A, 0, A, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 4096, None) == 1             # no trajectory rows
+    assert f(A, A, A, 1 << 31, A, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 4096, None) == 4       # overflow
+    assert f(A, A, A, 100, A, A, 1, 10, 10, 2, 1, 96, 0.0, A, A, A, 4096, None) == 2           # d = 96
+    assert f(A, A, A, 100, A, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 0, None) == 8              # workspace
+    sp = lib.vcs_shared_prefix
+    sp.restype = ctypes.c_int32
+    sp.argtypes = [ctypes.c_void_p] * 3 + [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_void_p] * 3
+    assert sp(A, A, A, -1, 10, A, None, None) == 1
+    assert sp(None, A, A, 2, 10, A, None, None) == 1
+    assert sp(A, A, A, 2, 1 << 31, A, None, None) == 4
+    fr = lib.vcs_attn_fwd_reuse
+    fr.restype = ctypes.c_int32
+    fr.argtypes = [ctypes.c_void_p] * 5 + [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 4 + \
+        [ctypes.c_float] + [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p]
+    assert fr(A, A, A, A, None, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 4096, None) == 1           # no shared map
+    assert fr(A, A, A, A, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 0, None) == 8                 # workspace
