@@ -200,7 +200,8 @@ __device__ __forceinline__ void issue_dq(uint32_t tmem_d, uint32_t dst_addr, uin
 
 // GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
 // tile (TMA gather4 with the 2-D maps tm_q/k/v, or tiled loads with the 3-D maps
-// tm_qr/kr/vr where a tile is one run of consecutive trajectory rows), and dK, dV are added
+// tm_qr/kr/vr and tm_qs/ks/vs, 128- and 32-row boxes, where a tile or a 32-row group is one
+// run of consecutive trajectory rows), and dK, dV are added
 // in fp32 to trajectory-layout accumulators (dk_acc, dv_acc) at row tok_gather[key];
 // otherwise segment-layout tiled loads, bf16 dK, dV, and tm_qr/kr/vr unused.
 template <int D, bool GATHER>
@@ -213,7 +214,9 @@ __global__ void __launch_bounds__(kThreads, 1)
              __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status,
              const int32_t* __restrict__ tok_gather, int32_t traj_tokens, float* __restrict__ dk_acc,
              float* __restrict__ dv_acc, const __grid_constant__ CUtensorMap tm_qr,
-             const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr) {
+             const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr,
+                    const __grid_constant__ CUtensorMap tm_qs, const __grid_constant__ CUtensorMap tm_ks,
+                    const __grid_constant__ CUtensorMap tm_vs) {
   using C = Bwd<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -278,9 +281,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
       }
       __syncwarp();
-      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &bars->kv_full, g, D, start + n * C::BM, end - 1,
+      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &tm_ks, &bars->kv_full, g, D, start + n * C::BM, end - 1,
                                    tok_gather, traj_tokens, status, lane);
-      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &bars->kv_full, g, D, start + n * C::BM, end - 1,
+      load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &tm_vs, &bars->kv_full, g, D, start + n * C::BM, end - 1,
                                    tok_gather, traj_tokens, status, lane);
       for (int it = 0; it < iters; ++it) {
         const int h = g * G + it / per_head;
@@ -300,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!__shfl_sync(0xffffffffu, go, 0)) break;
-        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q, &tm_q, &tm_qr, &bars->qdo_full, h, D, start + m * C::BN, end - 1,
+        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q, &tm_q, &tm_qr, &tm_qs, &bars->qdo_full, h, D, start + m * C::BN, end - 1,
                                      tok_gather, traj_tokens, status, lane);
       }
     } else if (lane == 0) {
@@ -636,7 +639,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
                   __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv, int32_t* status,
                   const int32_t* __restrict__ tok_gather, int32_t traj_tokens, float* __restrict__ dk_acc,
                   float* __restrict__ dv_acc, const __grid_constant__ CUtensorMap tm_qr,
-                  const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr) {
+                  const __grid_constant__ CUtensorMap tm_kr, const __grid_constant__ CUtensorMap tm_vr,
+                    const __grid_constant__ CUtensorMap tm_qs, const __grid_constant__ CUtensorMap tm_ks,
+                    const __grid_constant__ CUtensorMap tm_vs) {
   using C = D128;
   constexpr int D = C::D;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -715,9 +720,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         mbar_arrive_expect_tx(&bars->kv_full, 2 * C::TILE);
       }
       __syncwarp();
-      load_traj_tile<2, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
+      load_traj_tile<2, C::BLOCK>(smem + C::OFF_K, &tm_k, &tm_kr, &tm_ks, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
                                traj_tokens, status, lane);
-      load_traj_tile<2, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
+      load_traj_tile<2, C::BLOCK>(smem + C::OFF_V, &tm_v, &tm_vr, &tm_vs, &bars->kv_full, g, D, start + n * C::BM, end - 1, tok_gather,
                                traj_tokens, status, lane);
       for (int u = 0; u < U; ++u) {
         const int h = head_of(u);
@@ -736,7 +741,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           }
         }
         if (!__shfl_sync(0xffffffffu, go, 0)) break;
-        load_traj_tile<2, C::BLOCK>(qs, &tm_q, &tm_qr, &bars->q_full[stage], h, D, start + q0, end - 1, tok_gather, traj_tokens,
+        load_traj_tile<2, C::BLOCK>(qs, &tm_q, &tm_qr, &tm_qs, &bars->q_full[stage], h, D, start + q0, end - 1, tok_gather, traj_tokens,
                                  status, lane);
         if (lane == 0) {
           if (u >= C::NST && !mbar_wait(&bars->do_free[stage], ((u / C::NST) - 1) & 1)) {
@@ -1061,14 +1066,17 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
                                                          static_cast<const __nv_bfloat16*>(dout), rows, a.hq,
                                                          a.num_tokens, dvec, dq_acc);
   }
-  alignas(64) CUtensorMap tq, tk, tv, tdo, tqr, tkr, tvr;
+  alignas(64) CUtensorMap tq, tk, tv, tdo, tqr, tkr, tvr, tqs, tks, tvs;
   if (GATHER) {
     if (!encode_tma_rows_bf16(&tq, a.q, (uint64_t)a.hq * D, a.traj_tokens) ||
         !encode_tma_rows_bf16(&tk, a.k, (uint64_t)a.hkv * D, a.traj_tokens) ||
         !encode_tma_rows_bf16(&tv, a.v, (uint64_t)a.hkv * D, a.traj_tokens) ||
         !encode_tma_3d_bf16(&tqr, a.q, D, a.hq, a.traj_tokens, 64, 128) ||
         !encode_tma_3d_bf16(&tkr, a.k, D, a.hkv, a.traj_tokens, 64, 128) ||
-        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128))
+        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tqs, a.q, D, a.hq, a.traj_tokens, 64, 32) ||
+        !encode_tma_3d_bf16(&tks, a.k, D, a.hkv, a.traj_tokens, 64, 32) ||
+        !encode_tma_3d_bf16(&tvs, a.v, D, a.hkv, a.traj_tokens, 64, 32))
       return cudaErrorInvalidValue;
   } else if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
              !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
@@ -1101,7 +1109,8 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
           tq, tk, tv, tdo, tdq32, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv,
           a.scale, a.scale * 1.4426950408889634f, lse, dvec, static_cast<__nv_bfloat16*>(dk),
           static_cast<__nv_bfloat16*>(dv), a.status, a.tok_gather, (int32_t)a.traj_tokens, dk_t, dv_t,
-          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv);
+          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv, GATHER ? tqs : tq, GATHER ? tks : tk,
+          GATHER ? tvs : tv);
     } else {
       cudaError_t e =
           cudaFuncSetAttribute(bwd_main<D, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
@@ -1110,7 +1119,8 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
           tq, tk, tv, tdo, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, ntiles,
           a.scale, a.scale * 1.4426950408889634f, lse, dvec, dq_acc, static_cast<__nv_bfloat16*>(dk),
           static_cast<__nv_bfloat16*>(dv), a.status, a.tok_gather, (int32_t)a.traj_tokens, dk_t, dv_t,
-          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv);
+          GATHER ? tqr : tq, GATHER ? tkr : tk, GATHER ? tvr : tv, GATHER ? tqs : tq, GATHER ? tks : tk,
+          GATHER ? tvs : tv);
     }
   }
   auto convert = [&](const float* acc, void* out, int64_t elems) {

@@ -133,9 +133,10 @@ __device__ __forceinline__ int reuse_skip_rows(const int32_t* __restrict__ seg_s
 }
 
 // GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
-// tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr 3-D tiled
-// maps of the same tensors for tiles whose rows are one run of consecutive trajectory rows.
-// Otherwise tm_q/k/v are segment-layout tiled maps and tm_qr/kr/vr are unused.
+// tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr and
+// tm_qs/ks/vs 3-D tiled maps of the same tensors (128- and 32-row boxes) for tiles or
+// 32-row groups whose rows are consecutive trajectory rows.  Otherwise tm_q/k/v are
+// segment-layout tiled maps and the others are unused.
 template <int D, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -144,7 +145,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     int32_t npairs, float scale_log2, __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
                     int32_t* status, const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
                     const __grid_constant__ CUtensorMap tm_qr, const __grid_constant__ CUtensorMap tm_kr,
-                    const __grid_constant__ CUtensorMap tm_vr, const int32_t* __restrict__ seg_shared) {
+                    const __grid_constant__ CUtensorMap tm_vr, const int32_t* __restrict__ seg_shared,
+                    const __grid_constant__ CUtensorMap tm_qs, const __grid_constant__ CUtensorMap tm_ks,
+                    const __grid_constant__ CUtensorMap tm_vs) {
   using C = Fwd<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -218,10 +221,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(&bars->q_full, (has1 ? 2 : 1) * C::TILE);
         }
         __syncwarp();
-        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q0, &tm_q, &tm_qr, &bars->q_full, h, D, start + m0 * C::BM, end - 1,
+        load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q0, &tm_q, &tm_qr, &tm_qs, &bars->q_full, h, D, start + m0 * C::BM, end - 1,
                                      tok_gather, traj_tokens, status, lane);
         if (has1)
-          load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q1, &tm_q, &tm_qr, &bars->q_full, h, D, start + m1 * C::BM, end - 1,
+          load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_Q1, &tm_q, &tm_qr, &tm_qs, &bars->q_full, h, D, start + m1 * C::BM, end - 1,
                                        tok_gather, traj_tokens, status, lane);
         for (int c = 0; c < 2 * nkv; ++c) {
           const bool is_v = c == 2 * nkv - 1 || (c > 0 && (c & 1) == 0);
@@ -240,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (!__shfl_sync(0xffffffffu, go, 0)) break;
           load_traj_tile<C::KB, C::BLOCK>(smem + C::OFF_KV + slot * C::TILE, is_v ? &tm_v : &tm_k,
-                                          is_v ? &tm_vr : &tm_kr, &bars->kv_full[slot], g, D, start + j * C::BN,
+                                          is_v ? &tm_vr : &tm_kr, is_v ? &tm_vs : &tm_ks, &bars->kv_full[slot], g, D, start + j * C::BN,
                                           end - 1, tok_gather, traj_tokens, status, lane);
         }
       } else {
@@ -509,14 +512,17 @@ __global__ void __launch_bounds__(256) fwd_reuse_copy(const int32_t* __restrict_
 template <int D, bool GATHER>
 cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st) {
   using C = Fwd<D>;
-  alignas(64) CUtensorMap tq, tk, tv, tqr, tkr, tvr;
+  alignas(64) CUtensorMap tq, tk, tv, tqr, tkr, tvr, tqs, tks, tvs;
   if (GATHER) {
     if (!encode_tma_rows_bf16(&tq, a.q, (uint64_t)a.hq * D, a.traj_tokens) ||
         !encode_tma_rows_bf16(&tk, a.k, (uint64_t)a.hkv * D, a.traj_tokens) ||
         !encode_tma_rows_bf16(&tv, a.v, (uint64_t)a.hkv * D, a.traj_tokens) ||
         !encode_tma_3d_bf16(&tqr, a.q, D, a.hq, a.traj_tokens, 64, 128) ||
         !encode_tma_3d_bf16(&tkr, a.k, D, a.hkv, a.traj_tokens, 64, 128) ||
-        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128))
+        !encode_tma_3d_bf16(&tvr, a.v, D, a.hkv, a.traj_tokens, 64, 128) ||
+        !encode_tma_3d_bf16(&tqs, a.q, D, a.hq, a.traj_tokens, 64, 32) ||
+        !encode_tma_3d_bf16(&tks, a.k, D, a.hkv, a.traj_tokens, 64, 32) ||
+        !encode_tma_3d_bf16(&tvs, a.v, D, a.hkv, a.traj_tokens, 64, 32))
       return cudaErrorInvalidValue;
   } else if (!encode_tma_3d_bf16(&tq, a.q, D, a.hq, a.num_tokens, 64, 128) ||
              !encode_tma_3d_bf16(&tk, a.k, D, a.hkv, a.num_tokens, 64, 128) ||
@@ -544,7 +550,8 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
   attn_fwd_kernel<D, GATHER><<<grid, kThreads, C::SMEM, st>>>(
       tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
       static_cast<__nv_bfloat16*>(o), lse, a.status, a.tok_gather, (int32_t)a.traj_tokens, GATHER ? tqr : tq,
-      GATHER ? tkr : tk, GATHER ? tvr : tv, a.seg_shared);
+      GATHER ? tkr : tk, GATHER ? tvr : tv, a.seg_shared, GATHER ? tqs : tq, GATHER ? tks : tk,
+      GATHER ? tvs : tv);
   if (a.seg_shared != nullptr) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;

@@ -311,13 +311,15 @@ __device__ __forceinline__ void tma_gather4(void* dst, const void* map, uint64_t
 // row `last`) of one head from a trajectory-layout tensor through the gather map.  When the
 // tile's 128 rows are consecutive trajectory rows (inside a screenshot-and-text run of the
 // segment) lane 0 issues the KB tiled loads of the 3-D map tmap (box 64 x 1 head x 128 rows);
-// otherwise lane l gathers rows 4l .. 4l+3 of each 64-column block with the 2-D map gmap, to
-// the same swizzled positions.  Blocks are BLOCK bytes apart at dst.  A gather index outside
-// [0, traj_tokens) is recorded as a device check and read as row 0.  The caller has posted
-// the tile's bytes on `bar`.
+// otherwise each group of 8 lanes takes 32 rows: one tiled load of the 32-row map tmap32 if
+// they are consecutive (the text runs of the history), else lane l gathers rows 4l .. 4l+3
+// with the 2-D map gmap.  Every path puts a row where a tiled load of the whole tile would
+// (the 128-byte swizzle follows the shared-memory address).  Blocks are BLOCK bytes apart at
+// dst.  A gather index outside [0, traj_tokens) is recorded as a device check and read as
+// row 0.  The caller has posted the tile's bytes on `bar`.
 template <int KB, int BLOCK>
-__device__ __forceinline__ void load_traj_tile(uint8_t* dst, const void* gmap, const void* tmap, uint64_t* bar,
-                                               int head, int d, int s0, int last,
+__device__ __forceinline__ void load_traj_tile(uint8_t* dst, const void* gmap, const void* tmap, const void* tmap32,
+                                               uint64_t* bar, int head, int d, int s0, int last,
                                                const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
                                                int32_t* status, int lane) {
   int t[4];
@@ -338,6 +340,19 @@ __device__ __forceinline__ void load_traj_tile(uint8_t* dst, const void* gmap, c
     if (lane == 0) {
 #pragma unroll
       for (int kb = 0; kb < KB; ++kb) tma_load_3d(dst + kb * BLOCK, tmap, bar, kb * 64, head, base);
+    }
+    return;
+  }
+  const int g0 = lane & ~7;  // first lane of this lane's 32-row group
+  const int gbase = __shfl_sync(0xffffffffu, t[0], g0);
+  bool grun = s0 + 4 * g0 + 31 <= last;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) grun = grun && t[i] == gbase + 4 * (lane - g0) + i;
+  const unsigned votes = __ballot_sync(0xffffffffu, grun);
+  if (((votes >> g0) & 0xffu) == 0xffu) {
+    if (lane == g0) {
+#pragma unroll
+      for (int kb = 0; kb < KB; ++kb) tma_load_3d(dst + kb * BLOCK + g0 * 512, tmap32, bar, kb * 64, head, gbase);
     }
   } else {
 #pragma unroll
