@@ -209,9 +209,9 @@ class Path:
         self.bwd_ws = T(self.bwd_ws_bytes, dt=torch.uint8)
         self.launches_per_step = 0
 
-    def step(self, tstream, ev=None, before_chunk=None, after_chunk=None):
+    def step(self, tstream, ev=None, before_chunk=None, after_chunk=None, before_bwd=None):
         """One pass of the hot path over all chunks; optional per-chunk events appended to ev and
-        hooks called before a chunk's first launch and after its last one."""
+        hooks called before a chunk's first launch, before its backward and after its last one."""
         vcs, w = self.vcs, self.w
         stream = tstream.cuda_stream
         hq, hkv, d = w.hq, w.hkv, w.d
@@ -252,6 +252,8 @@ class Path:
             if evs:
                 evs[4].record(tstream)
             dout = self.dout[ci["tok0"]:ci["tok1"]]
+            if before_bwd is not None:
+                before_bwd(i)
             st = vcs.vcs_attn_bwd(self.q, self.k, self.v, self.o, self.lse, dout, self.cu_seqlens, nseg, ntok,
                                   ci["max_seqlen"], hq, hkv, d, 0.0, self.dq, self.dk, self.dv, self.bwd_ws,
                                   self.bwd_ws_bytes, stream)
@@ -643,10 +645,12 @@ def run_e2e(path, args, flops, stream):
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     # Each step's inputs are copied from pinned host memory on a second stream, chunk by
     # chunk: a chunk's copy for the next step starts once its launches of this step are done,
-    # so it overlaps the other chunk's compute; the compute of a chunk waits for its copy.
+    # so it overlaps the other chunk's compute.  A chunk's builder, gather and forward wait
+    # for its Q/K/V; its backward for its dO (copied after them, under the forward).
     cs = torch.cuda.Stream(device=path.dev)
     nch = len(path.chunk_in)
     copied = [torch.cuda.Event() for _ in range(nch)]
+    copied_do = [torch.cuda.Event() for _ in range(nch)]
     done = [torch.cuda.Event() for _ in range(nch)]
     state = {"step": 0}
 
@@ -657,11 +661,15 @@ def run_e2e(path, args, flops, stream):
             path.q_traj[a:b].copy_(host["q"][a:b], non_blocking=True)
             path.k_traj[a:b].copy_(host["k"][a:b], non_blocking=True)
             path.v_traj[a:b].copy_(host["v"][a:b], non_blocking=True)
-            path.dout[t0_:t1_].copy_(host["do"][t0_:t1_], non_blocking=True)
             copied[i].record(cs)
+            path.dout[t0_:t1_].copy_(host["do"][t0_:t1_], non_blocking=True)
+            copied_do[i].record(cs)
 
     def before(i):
         stream.wait_event(copied[i])
+
+    def before_bwd(i):
+        stream.wait_event(copied_do[i])
 
     def after(i):
         done[i].record(stream)
@@ -678,7 +686,7 @@ def run_e2e(path, args, flops, stream):
         copy_chunk(i)
     for s_ in range(args.steps):
         state["step"] = s_
-        path.step(stream, before_chunk=before, after_chunk=after)
+        path.step(stream, before_chunk=before, after_chunk=after, before_bwd=before_bwd)
         # result read back: the last chunk's log-sum-exp (the loss-side statistic)
         res.copy_(path.lse.view(-1)[: res.numel()], non_blocking=True)
     t1.record(stream)
