@@ -297,6 +297,34 @@ def oracle_sample(w, window, keep, seconds_hint=True):
     return flops / (t_build + t_attn) / 1e12, sample, t_build + t_attn
 
 
+def rank_workload(w, rank: int):
+    """The batch rank `rank` lays out: segments of different trajectories are independent, so
+    ranks shard the units with no data-path exchange: every rank draws its own batch of the
+    workload (same sizes and distributions, its own seed) and the job processes world x batch."""
+    import dataclasses
+    return w if rank == 0 else dataclasses.replace(w, seed=w.seed + 7919 * rank)
+
+
+def max_over_ranks(value: float, device) -> float:
+    """The slowest rank's time (the job's time), over the default process group if there is one."""
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, device) -> float:
+    """The job's total of a per-rank quantity (flops, tokens), over the default process group."""
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
 def run_reference(args, w, window, keep, rank, world):
     if rank != 0:
         return
@@ -358,7 +386,7 @@ def main():
         v, sample, _ = oracle_sample(w, window, keep)
         cpu = {"value": v, "unit": "TFLOP/s", "cores": os.cpu_count(), "kind": "oracle", "sample": sample}
 
-    path = Path(w, window, keep, dev)
+    path = Path(rank_workload(w, rank), window, keep, dev)
     stream = torch.cuda.current_stream()
     flops, f_fwd, f_bwd = credited_flops(path.seg_lens, w.hq, w.d)
     for _ in range(args.warmup):
@@ -385,10 +413,7 @@ def main():
     barrier()
     ck = clocks.stop()
     ms = t0.elapsed_time(t1) / args.steps
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, dev)
     # per chunk: [0]-[1] build, (host reads the sizes), [2]-[3] gather, [3]-[4] fwd, [4]-[5] bwd
     build_ms = sum(e[0].elapsed_time(e[1]) for e, _ in ev) / args.steps
     gather_ms = sum(e[2].elapsed_time(e[3]) for e, _ in ev) / args.steps
@@ -398,14 +423,16 @@ def main():
     gather_bytes = path.num_tokens * 2 * (w.hq + 2 * w.hkv) * w.d * 2     # rows read once + written once
     bwd_launch_flops = f_bwd / len(path.chunk_in)
 
-    value = flops * world / (ms / 1e3) / 1e12
+    job_flops = sum_over_ranks(flops, dev)               # every rank's own batch
+    job_tokens = sum_over_ranks(float(path.num_tokens), dev)
+    value = job_flops / (ms / 1e3) / 1e12
     burst, sustained, hbm, src = peaks()
 
     # end to end through the public API with host buffers: pinned host -> device copies of the
     # step's inputs and a device -> host read of its result, inside the timed region
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(path, args, flops * world, stream)
+        e2e = run_e2e(path, args, job_flops, stream)
 
     next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
     fused = None if args.no_fused else run_fused(path, stream)
@@ -427,7 +454,7 @@ def main():
         "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,
         "frac_of_bf16_burst": value / burst, "frac_of_bf16_sustained": value / sustained,
         "flash_convention_tflops": value * 14.0 / 12.0,
-        "segment_tokens_per_s": path.num_tokens * world / (ms / 1e3),
+        "segment_tokens_per_s": job_tokens / (ms / 1e3),
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
                      "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s", "frac": ach_bwd / sustained,
                      "peak_source": f"{src} bf16 sustained",
@@ -631,17 +658,21 @@ def run_e2e(path, args, flops, stream):
         avail = int(next(l for l in open("/proc/meminfo") if l.startswith("MemAvailable")).split()[1]) * 1024
     except Exception:
         avail = 0
-    if need > 0.6 * avail:
+    # every rank takes the same branch (the decisions are reduced over ranks), so that the
+    # collectives below are entered by all of them or by none
+    if sum_over_ranks(float(need > 0.6 * avail), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s",
                 "error": f"pinned staging of {need / 2**30:.0f} GiB exceeds 60% of available host memory"}
-    host = {}
+    host, err = {}, None
     try:
         for name, t in srcs.items():
             host[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
             host[name].copy_(t)
         res = torch.empty(path.w.hq * path.max_tok, dtype=torch.float32, pin_memory=True)
     except RuntimeError as e:
-        return {"value": None, "unit": "TFLOP/s", "error": f"pinned staging failed: {e}"[:200]}
+        err = f"pinned staging failed: {e}"[:200]
+    if sum_over_ranks(float(err is not None), path.dev) > 0:
+        return {"value": None, "unit": "TFLOP/s", "error": err or "pinned staging failed on another rank"}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     # Each step's inputs are copied from pinned host memory on a second stream, chunk by
     # chunk: a chunk's copy for the next step starts once its launches of this step are done,
@@ -692,7 +723,7 @@ def run_e2e(path, args, flops, stream):
     t1.record(stream)
     torch.cuda.synchronize()
     d2h = res.numel() * 4
-    ms = t0.elapsed_time(t1) / args.steps
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, path.dev)
     return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
