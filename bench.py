@@ -41,6 +41,7 @@ from paper_2607_11185_gb300 import workloads  # noqa: E402
 
 METRIC = "segmented attn fwd+bwd TFLOP/s & % BF16 peak; segment tokens/s; vs CPU oracle"
 CHUNK_BYTES = 130 << 30   # per-chunk working set budget on the device (fewer, larger launches)
+NOMINAL_BF16_TFLOPS = 2250.0  # GB300 dense bf16 tensor rate as NVIDIA quotes it (2:4-sparse figures are 2x)
 
 
 def peaks():
@@ -359,6 +360,7 @@ def main():
     ap.add_argument("--no-next-rows", action="store_true", help="skip the stream-field / loss kernel timings")
     ap.add_argument("--no-fused", action="store_true", help="skip the gathered-attention (fused gather) timing")
     ap.add_argument("--no-reuse", action="store_true", help="skip the prefix-reuse forward timing")
+    ap.add_argument("--no-hbm-kernels", action="store_true", help="skip the builder / gather timings")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -437,6 +439,7 @@ def main():
     next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
     fused = None if args.no_fused else run_fused(path, stream)
     reuse = None if args.no_reuse else run_reuse(path, stream)
+    hbm_kernels = None if args.no_hbm_kernels else run_hbm_kernels(path, stream, hbm)
 
     ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
     line = {
@@ -453,6 +456,7 @@ def main():
         "attn_fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "attn_bwd_tflops": f_bwd / (bwd_ms / 1e3) / 1e12,
         "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,
         "frac_of_bf16_burst": value / burst, "frac_of_bf16_sustained": value / sustained,
+        "frac_of_bf16_nominal": value / NOMINAL_BF16_TFLOPS,
         "flash_convention_tflops": value * 14.0 / 12.0,
         "segment_tokens_per_s": job_tokens / (ms / 1e3),
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
@@ -465,6 +469,7 @@ def main():
         "next_rows": next_rows,
         "fused_gather": fused,
         "prefix_reuse": reuse,
+        "hbm_kernels": hbm_kernels,
         "gpu_launches": path.launches_per_step * args.steps,
         "clocks": ck,
     }
@@ -530,6 +535,76 @@ def run_next_rows(path, stream, hbm_gbs):
         gbs = nbytes / (ms / 1e3) / 1e9
         out[name] = {"ms": ms, "bytes": int(nbytes), "gbs": gbs, "frac_of_hbm": gbs / hbm_gbs}
     assert int(status.item()) == 0 and int(lws[:4].view(torch.int32).item()) == 0
+    return out
+
+
+def _median_ms(fn, stream, flush, reps=10, warm=3):
+    """Median of `reps` launches of fn (after `warm`), L2 flushed before each (CUDA events)."""
+    times = []
+    for i in range(warm + reps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        assert fn() == 0
+        e1.record(stream)
+        if i >= warm:
+            times.append((e0, e1))
+    torch.cuda.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in times)
+
+
+def run_hbm_kernels(path, stream, hbm_gbs, stress_traj=4096):
+    """Builder and gather timed alone (L2 flushed, 3 warm-up + median of 10): the builder on the
+    largest chunk and on a 4,096-trajectory batch of the same step distribution (a size at
+    which the builder's writes, not its launches, take the time), the gather on the largest
+    chunk.  Algorithmic bytes: the builder writes 13 B per segment token (gather index, source
+    step, position, loss mask) and 8 B per segment, and reads 8 B per step; the gather reads
+    and writes 2 (Hq + 2 Hkv) d bytes per segment token."""
+    vcs, w = path.vcs, path.w
+    sp = stream.cuda_stream
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=path.dev)
+    out = {"l2": "flushed (256 MB write) before every timed launch"}
+    ci = path.chunk_in[0]
+    nseg, ntok = ci["s1"] - ci["s0"], ci["tok1"] - ci["tok0"]
+
+    def build(c, b, nsteps, img, txt, cu_seqlens, seg_traj, gi, src, pos, mask, sizes, ws, nb, ms, mt):
+        return lambda: vcs.vcs_build_segments(c, b, nsteps, img, txt, path.window, path.keep, ms, mt, cu_seqlens,
+                                              seg_traj, gi, src, pos, mask, sizes, ws, nb, sp)
+
+    seg_traj = torch.empty(path.max_seg, dtype=torch.int32, device=path.dev)
+    ms = _median_ms(build(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"], path.cu_seqlens,
+                          seg_traj, path.tok_gather, path.tok_src, path.tok_pos, path.tok_mask, path.sizes,
+                          path.seg_ws, path.seg_ws_bytes, path.max_seg, path.max_tok), stream, flush)
+    nbytes = 13 * ntok + 8 * nseg + 8 * ci["nsteps"]
+    out["builder"] = {"us": ms * 1e3, "segment_tokens": ntok, "bytes": nbytes,
+                      "gbs": nbytes / (ms / 1e3) / 1e9}
+    # builder stress: 4,096 trajectories drawn like the workload's (its own seed)
+    import dataclasses
+    ws_ = dataclasses.replace(w, num_traj=stress_traj, seed=w.seed + 4096)
+    cu, img, txt = workloads.draw_steps(ws_)
+    seg_lens, _ = layout_stats(cu, img, txt, path.window, path.keep)
+    S, N = int(len(seg_lens)), int(seg_lens.sum())
+    if N < 2 ** 31 - 1 and N * 13 < (24 << 30):
+        dev = path.dev
+        T = lambda n, dt=torch.int32: torch.empty(max(n, 1), dtype=dt, device=dev)  # noqa: E731
+        d_cu, d_img, d_txt = (torch.from_numpy(np.ascontiguousarray(x, dtype=np.int32)).to(dev) for x in (cu, img, txt))
+        nb = vcs.vcs_segments_workspace_size(stress_traj, len(img))
+        bufs = [T(S + 1), T(S), T(N), T(N), T(N), T(N, torch.uint8), torch.zeros(3, dtype=torch.int64, device=dev),
+                T(nb, torch.uint8)]
+        ms = _median_ms(build(d_cu, stress_traj, len(img), d_img, d_txt, *bufs[:7], bufs[7], nb, S, N), stream,
+                        flush)
+        nbytes = 13 * N + 8 * S + 8 * len(img)
+        out["builder_stress"] = {"trajectories": stress_traj, "segments": S, "segment_tokens": N, "us": ms * 1e3,
+                                 "bytes": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9,
+                                 "frac_of_hbm": nbytes / (ms / 1e3) / 1e9 / hbm_gbs}
+        del bufs
+    qt, kt, vt = (x[ci["ttok0"]:ci["ttok1"]] for x in (path.q_traj, path.k_traj, path.v_traj))
+    ms = _median_ms(lambda: vcs.vcs_gather(qt, kt, vt, ci["ttok1"] - ci["ttok0"], path.tok_gather, ntok, w.hq, w.hkv,
+                                           w.d, path.q, path.k, path.v, path.gstatus, sp), stream, flush)
+    nbytes = ntok * 2 * (w.hq + 2 * w.hkv) * w.d * 2
+    out["gather"] = {"ms": ms, "bytes": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9,
+                     "frac_of_hbm": nbytes / (ms / 1e3) / 1e9 / hbm_gbs}
+    assert path.device_status() == (0, 0, 0)
     return out
 
 

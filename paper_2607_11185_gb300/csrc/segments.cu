@@ -21,8 +21,9 @@
 //                   capacity checks, the vcs_sizes record
 //   seg_write       one thread per trajectory: cu_seqlens, seg_traj and the
 //                   per-segment step bounds used by the expansion
-//   seg_expand      grid-stride over segment tokens: gather index, source
-//                   step, position, loss mask (two binary searches per token)
+//   seg_expand      one warp per 4,096 segment tokens: gather index, source
+//                   step, position, loss mask, streamed run by run (one run per
+//                   step of the segment), 32 consecutive tokens per store
 #include <climits>
 #include <cstdint>
 
@@ -259,34 +260,58 @@ __device__ __forceinline__ int64_t last_le(const int64_t* __restrict__ arr, int6
   return lo;
 }
 
+// One warp per chunk of kExpandChunk consecutive segment tokens.  A segment is a sequence of
+// runs, one per step: the response tokens of each step before a_j (text-only history), then
+// the screenshot-and-response tokens of each step a_j..e_j; inside a run the gather index,
+// the position and the mask follow from the run's start, so the warp finds the run of its
+// first token once (two binary searches, uniform across the lanes) and then streams the runs
+// in order, the lanes writing 32 consecutive tokens per store.
+constexpr int kExpandChunk = 4096;
+
 __global__ void __launch_bounds__(256) seg_expand(const int32_t* __restrict__ step_img,
                                                   int32_t* __restrict__ tok_gather, int32_t* __restrict__ tok_src_step,
                                                   int32_t* __restrict__ tok_pos, uint8_t* __restrict__ tok_loss_mask,
                                                   SegWorkspace w) {
   if (w.totals[3] != 0) return;
   const int64_t nseg = w.totals[0], ntok = w.totals[1];
-  for (int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; n < ntok; n += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t seg = last_le(w.seg_start, 0, nseg - 1, n);
-    const int64_t p = n - w.seg_start[seg];
-    const int64_t g0 = w.seg_first[seg], A = w.seg_full[seg], S = w.seg_new[seg], E = w.seg_last[seg];
-    const int64_t t0 = w.txt_pre[g0];
-    const int64_t H = w.txt_pre[A] - t0;  // text-only history (steps before a_j)
-    int64_t gather, u;
-    uint8_t m;
-    if (p < H) {
-      const int64_t target = t0 + p;
-      u = last_le(w.txt_pre, g0, A - 1, target);
-      gather = w.step_off[u] + step_img[u] + (target - w.txt_pre[u]);
-      m = 0;
-    } else {
-      gather = w.step_off[A] + (p - H);  // full steps a_j..e_j are contiguous in the trajectory
-      u = last_le(w.step_off, A, E, gather);
-      m = (u >= S && gather >= w.step_off[u] + step_img[u]) ? 1 : 0;
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t c = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); c * kExpandChunk < ntok;
+       c += warps) {
+    int64_t n = c * kExpandChunk;
+    const int64_t nend = min(n + (int64_t)kExpandChunk, ntok);
+    int64_t seg = last_le(w.seg_start, 0, nseg - 1, n);
+    while (n < nend) {
+      while (w.seg_start[seg + 1] <= n) ++seg;  // skip segments without tokens
+      const int64_t start = w.seg_start[seg], next = w.seg_start[seg + 1];
+      const int64_t g0 = w.seg_first[seg], A = w.seg_full[seg], S = w.seg_new[seg], E = w.seg_last[seg];
+      const int64_t t0 = w.txt_pre[g0], H = w.txt_pre[A] - t0, f0 = w.step_off[A];
+      // the run (step u) of position p = n - start, and its bounds [lo, hi) in the segment
+      const int64_t p = n - start;
+      int64_t u = p < H ? last_le(w.txt_pre, g0, A - 1, t0 + p) : last_le(w.step_off, A, E, f0 + (p - H));
+      const int64_t send = min(next, nend);
+      while (n < send) {
+        const bool hist = u < A;
+        const int64_t lo = hist ? w.txt_pre[u] - t0 : H + (w.step_off[u] - f0);
+        const int64_t hi = hist ? w.txt_pre[u + 1] - t0 : H + (w.step_off[u + 1] - f0);
+        const int64_t img = step_img[u];
+        // token at position q of the run's step: history tokens are the step's response
+        // tokens (after its screenshot); a full step's tokens start with the screenshot
+        const int64_t g_base = hist ? w.step_off[u] + img - lo : w.step_off[u] - lo;
+        const bool trainable_step = !hist && u >= S;
+        const int64_t rend = min(start + hi, send);
+        for (int64_t m = n + lane; m < rend; m += 32) {
+          const int64_t q = m - start;
+          tok_gather[m] = (int32_t)(g_base + q);
+          tok_src_step[m] = (int32_t)u;
+          tok_pos[m] = (int32_t)q;
+          if (tok_loss_mask != nullptr) tok_loss_mask[m] = (trainable_step && q - lo >= img) ? 1 : 0;
+        }
+        n = max(n, rend);
+        ++u;
+      }
+      ++seg;
     }
-    tok_gather[n] = (int32_t)gather;
-    tok_src_step[n] = (int32_t)u;
-    tok_pos[n] = (int32_t)p;
-    if (tok_loss_mask != nullptr) tok_loss_mask[n] = m;
   }
 }
 
@@ -352,7 +377,7 @@ cudaError_t launch_seg_build(const int32_t* cu_steps, int32_t num_traj, int32_t 
   const int tb = 128;
   const int nb = num_traj > 0 ? (num_traj + tb - 1) / tb : 1;
   seg_write<<<nb, tb, 0, st>>>(cu_steps, num_traj, window, keep, cu_seqlens, seg_traj, w);
-  seg_expand<<<152 * 8, 256, 0, st>>>(step_img, tok_gather, tok_src_step, tok_pos, tok_loss_mask, w);
+  seg_expand<<<152 * 16, 256, 0, st>>>(step_img, tok_gather, tok_src_step, tok_pos, tok_loss_mask, w);
   return cudaGetLastError();
 }
 
