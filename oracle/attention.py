@@ -4,7 +4,7 @@ The paper trains its policy with the segments that Algorithm 1 emits
 (Sec. 3.4; the actor-update and reference-policy phases of App. C.2); it does
 not spell the attention out.  What is computed here is the plain definition
 of causal softmax self-attention restricted to one segment, with grouped
-query heads, read as follows (the design doc lists these readings):
+query heads, read as follows:
 
   token i of segment sigma(i) at in-segment position p(i), query head h,
   key/value head g(h) = floor(h * Hkv / Hq):

@@ -11,8 +11,7 @@ with group-relative advantage A_ij shared by every segment of that rollout,
 rho_t = pi_theta(a_t | x_<t) / pi_rollout(a_t | x_<t), asymmetric clipping
 eps_l = 0.2, eps_h = 0.28 (DAPO), a clip-ratio cap c = 3.0 and a KL weight
 lambda = 1e-4.  The paper gives no formula for the cap or the KL estimator and
-no normaliser beyond the expectations; this oracle reads them as follows (the
-same readings are listed in the design doc):
+no normaliser beyond the expectations; this oracle reads them as follows:
 
   * cap: dual clipping for negative advantages, the objective of a token with
     A < 0 is max(min(rho A, clip(rho) A), c A);

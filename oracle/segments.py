@@ -10,7 +10,7 @@ Two independent builders of the same segmentation:
   takes K + delta new steps, every later one delta new steps, and retains the
   K most recent earlier steps with their screenshots.
 
-Readings where the paper is silent (listed in the design doc as well):
+Readings where the paper is silent:
   * the step model: step t contributes img[t] screenshot tokens followed by
     txt[t] response tokens; the screenshot of step 1 is the initial
     observation and every screenshot increments ``n_img`` (also zero-token
