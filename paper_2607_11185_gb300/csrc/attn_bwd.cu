@@ -1090,15 +1090,12 @@ cudaError_t launch_bwd_d(const AttnArgs& a, const void* o, const float* lse, con
   dim3 grid((unsigned)ntiles, (unsigned)(gx < 65535 ? gx : 65535), (unsigned)((gx + 65534) / 65535));
   if (ntiles > 0) {
     if (D == 128) {
-      // the warpgroups' setmaxnreg targets are served from the registers the
-      // block is launched with: refuse to launch a build that got fewer
-      static int regs_ok = -1;
-      if (regs_ok < 0) {
-        cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, bwd_main_d128<GATHER>);
-        if (e != cudaSuccess) return e;
-        regs_ok = fa.numRegs == D128::REG_LAUNCH ? 1 : 0;
-      }
+      static std::atomic<int> regs_cache{-1};
+      bool regs_ok = false;
+      if (cudaError_t e = launch_regs_match(reinterpret_cast<const void*>(bwd_main_d128<GATHER>), D128::REG_LAUNCH,
+                                            &regs_cache, &regs_ok);
+          e != cudaSuccess)
+        return e;
       if (!regs_ok) return cudaErrorInvalidConfiguration;
       alignas(64) CUtensorMap tdq32;  // fp32 accumulator, [128 rows][32 dims] boxes, 128-byte swizzle
       if (!encode_tma_3d_f32(&tdq32, dq_acc, D, a.hq, a.num_tokens, 32, 128, true)) return cudaErrorInvalidValue;

@@ -529,15 +529,12 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
              !encode_tma_3d_bf16(&tv, a.v, D, a.hkv, a.num_tokens, 64, 128)) {
     return cudaErrorInvalidValue;
   }
-  // the warpgroups' setmaxnreg targets are served from the registers the block
-  // is launched with: refuse to launch a build that got a different count
-  static int regs_ok = -1;
-  if (regs_ok < 0) {
-    cudaFuncAttributes fa;
-    cudaError_t e = cudaFuncGetAttributes(&fa, attn_fwd_kernel<D, GATHER>);
-    if (e != cudaSuccess) return e;
-    regs_ok = fa.numRegs == kRegLaunch ? 1 : 0;
-  }
+  static std::atomic<int> regs_cache{-1};
+  bool regs_ok = false;
+  if (cudaError_t e = launch_regs_match(reinterpret_cast<const void*>(attn_fwd_kernel<D, GATHER>), kRegLaunch,
+                                        &regs_cache, &regs_ok);
+      e != cudaSuccess)
+    return e;
   if (!regs_ok) return cudaErrorInvalidConfiguration;
   cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;

@@ -2,6 +2,7 @@
 // kernel translation units.  Not part of the public interface.
 #pragma once
 
+#include <atomic>
 #include <cstddef>
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -92,14 +93,31 @@ cudaError_t launch_shared_prefix(const int32_t* cu_seqlens, const int32_t* seg_t
 bool encode_tma_3d_bf16(void* map /*CUtensorMap*/, const void* base, uint64_t d, uint64_t heads, uint64_t tokens,
                         uint32_t box_d, uint32_t box_rows);
 
-// fp32 variant (bulk reduce-add targets): no swizzle, or the 128-byte swizzle
-// (box_d * 4 must then be 128).
 // 2-D map over a row-major [rows, row_elems] bf16 tensor with a 64-column x 1-row box and the
 // 128-byte swizzle: the map of the TMA gather4 loads (one row per gathered token)
 bool encode_tma_rows_bf16(void* map, const void* base, uint64_t row_elems, uint64_t rows);
+// fp32 variant of encode_tma_3d_bf16 (bulk reduce-add targets): no swizzle, or the 128-byte
+// swizzle (box_d * 4 must then be 128).
 bool encode_tma_3d_f32(void* map, const void* base, uint64_t d, uint64_t heads, uint64_t tokens, uint32_t box_d,
                        uint32_t box_rows, bool swizzle128 = false);
 
 constexpr size_t kWsHeader = 256;  // attention workspace header (status word first)
+
+// Whether kernel fn was built with exactly `want` registers per thread: a kernel whose
+// warpgroups move registers with setmaxnreg is served from the registers its block is launched
+// with, so a build that got another count must not run.  The answer is cached in *cache
+// (-1 until first asked); concurrent first calls from several host threads are safe.
+inline cudaError_t launch_regs_match(const void* fn, int want, std::atomic<int>* cache, bool* ok) {
+  int c = cache->load(std::memory_order_relaxed);
+  if (c < 0) {
+    cudaFuncAttributes fa;
+    const cudaError_t e = cudaFuncGetAttributes(&fa, fn);
+    if (e != cudaSuccess) return e;
+    c = fa.numRegs == want ? 1 : 0;
+    cache->store(c, std::memory_order_relaxed);
+  }
+  *ok = c == 1;
+  return cudaSuccess;
+}
 
 }  // namespace vcs
