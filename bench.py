@@ -156,11 +156,11 @@ def make_chunks(seg_lens, seg_traj, num_traj, hq, hkv, d):
 class Path:
     """Device-resident inputs and per-chunk buffers for the hot path."""
 
-    def __init__(self, w: workloads.Workload, window: int, keep: int, device):
+    def __init__(self, w: workloads.Workload, window: int, keep: int, device, steps=None):
         from paper_2607_11185_gb300 import vcs
         self.vcs = vcs
         self.w, self.window, self.keep, self.dev = w, window, keep, device
-        cu, img, txt = workloads.draw_steps(w)
+        cu, img, txt = workloads.draw_steps(w) if steps is None else steps
         self.cu, self.img, self.txt = cu, img, txt
         self.seg_lens, self.seg_traj = layout_stats(cu, img, txt, window, keep)
         self.num_tokens = int(self.seg_lens.sum())
@@ -170,7 +170,7 @@ class Path:
         # resident inputs: step counts, trajectory Q/K/V, upstream gradient dO (segment layout)
         self.q_traj, self.k_traj, self.v_traj = workloads.draw_traj_qkv(w, self.ntraj_tok, device=device)
         self.dout = workloads.draw_dout(w, self.num_tokens, device=device)
-        self.chunks = make_chunks(self.seg_lens, self.seg_traj, w.num_traj, w.hq, w.hkv, w.d)
+        self.chunks = make_chunks(self.seg_lens, self.seg_traj, len(cu) - 1, w.hq, w.hkv, w.d)
         self.chunk_in = []
         seg_cum = np.concatenate([[0], np.cumsum(self.seg_lens)])
         max_tok = max_seg = max_steps = 0
@@ -335,12 +335,42 @@ def oracle_one_core(d: int, rows: int, seed: int):
             "sample": f"fp64 attention fwd+bwd of 1 query head over a {rows}-token segment, BLAS on one thread"}
 
 
-def rank_workload(w, rank: int):
-    """The batch rank `rank` lays out: segments of different trajectories are independent, so
-    ranks shard the units with no data-path exchange: every rank draws its own batch of the
-    workload (same sizes and distributions, its own seed) and the job processes world x batch."""
+def lpt_partition(costs, world: int):
+    """Longest-processing-time assignment of units to ranks: the units in order of decreasing
+    cost, each to the rank with the least cost so far (the lowest rank on ties).  Returns each
+    rank's unit indices in increasing order."""
+    order = sorted(range(len(costs)), key=lambda i: (-costs[i], i))
+    load = [0.0] * world
+    parts = [[] for _ in range(world)]
+    for i in order:
+        r = min(range(world), key=lambda j: (load[j], j))
+        parts[r].append(i)
+        load[r] += costs[i]
+    return [sorted(p) for p in parts]
+
+
+def rank_batch(w, window: int, keep: int, rank: int, world: int):
+    """The trajectories rank `rank` runs, as (cu_steps, step_img, step_txt, global indices).
+
+    Segments of different trajectories are independent, so ranks shard trajectories with no
+    data-path exchange.  The job draws the workload's distribution for world x its trajectory
+    count (the first w.num_traj trajectories are exactly the one-GPU batch) and splits them by
+    longest processing time on each trajectory's attention cost, the sum over its segments of
+    L(L+1)/2 causal pairs: weak scaling, each rank getting about one workload's worth."""
     import dataclasses
-    return w if rank == 0 else dataclasses.replace(w, seed=w.seed + 7919 * rank)
+    cu, img, txt = workloads.draw_steps(dataclasses.replace(w, num_traj=w.num_traj * world))
+    ntraj = len(cu) - 1
+    if world == 1:
+        return cu, img, txt, list(range(ntraj))
+    seg_lens, seg_traj = layout_stats(cu, img, txt, window, keep)
+    cost = np.zeros(ntraj)
+    np.add.at(cost, seg_traj, (seg_lens * (seg_lens + 1) // 2).astype(np.float64))
+    mine = lpt_partition(cost.tolist(), world)[rank]
+    steps = [(int(cu[b]), int(cu[b + 1])) for b in mine]
+    rcu = np.concatenate([[0], np.cumsum([g1 - g0 for g0, g1 in steps])]).astype(np.int32)
+    rimg = np.concatenate([img[g0:g1] for g0, g1 in steps] or [np.zeros(0, np.int32)]).astype(np.int32)
+    rtxt = np.concatenate([txt[g0:g1] for g0, g1 in steps] or [np.zeros(0, np.int32)]).astype(np.int32)
+    return rcu, rimg, rtxt, mine
 
 
 def max_over_ranks(value: float, device) -> float:
@@ -424,7 +454,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample(w, window, keep)
 
-    path = Path(rank_workload(w, rank), window, keep, dev)
+    path = Path(w, window, keep, dev, steps=rank_batch(w, window, keep, rank, world)[:3])
     stream = torch.cuda.current_stream()
     flops, f_fwd, f_bwd = credited_flops(path.seg_lens, w.hq, w.d)
     for _ in range(args.warmup):
@@ -485,7 +515,10 @@ def main():
         "config": {"workload": w.name, "window": window, "keep": keep, "num_traj": w.num_traj, "hq": w.hq,
                    "hkv": w.hkv, "d": w.d, "segments": int(len(path.seg_lens)), "segment_tokens": path.num_tokens,
                    "max_seqlen": int(path.seg_lens.max()), "chunks": len(path.chunk_in),
-                   "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)"},
+                   "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)",
+                   **({"sharding": f"{world * w.num_traj} trajectories over {world} ranks by longest processing "
+                                   f"time on sum L(L+1)/2; segments, tokens and chunks above are rank 0's"}
+                      if world > 1 else {})},
         "attn_tflop_credited": flops / 1e12,
         "builder_ms": build_ms, "gather_ms": gather_ms, "gather_gbs": gather_bytes / (gather_ms / 1e3) / 1e9,
         "attn_fwd_ms": fwd_ms, "attn_bwd_ms": bwd_ms,

@@ -1,11 +1,13 @@
 """The bench's multi-rank host logic on CPU (gloo, world size 2, no GPU).
 
 Segments of different trajectories are independent, so ranks shard the units with no
-data-path exchange: each rank lays out its own batch of the workload, the job's time is the
-slowest rank's, its flops and tokens the sum over ranks, and a decision that guards a
-collective is reduced over ranks so that every rank takes the same branch.
+data-path exchange: the job draws world x the workload's trajectories and each rank takes its
+longest-processing-time share by attention cost, the job's time is the slowest rank's, its flops
+and tokens the sum over ranks, and a decision that guards a collective is reduced over ranks so
+that every rank takes the same branch.
 """
 import contextlib
+import dataclasses
 import io
 import os
 import socket
@@ -41,11 +43,13 @@ def _worker(rank, world, port, out):
             # a guard that only one rank would fail is seen as failed by both
             "guard": bench.sum_over_ranks(float(rank == 1), dev),
         }
-        w = bench.rank_workload(workloads.WORKLOADS["traj8_w3"], rank)
-        cu, img, txt = workloads.draw_steps(w)
-        res["seed"] = w.seed
+        w = workloads.WORKLOADS["traj8_w3"]
+        cu, img, txt, mine = bench.rank_batch(w, w.window, w.keep, rank, world)
+        res["traj"] = mine
         res["steps"] = int(cu[-1])
         res["img_sum"] = int(img.sum())
+        lens, _ = bench.layout_stats(cu, img, txt, w.window, w.keep)
+        res["cost"] = float((lens * (lens + 1) // 2).sum())
         # the reference arm: only rank 0 runs and prints (the oracle is not run elsewhere)
         if rank == 1:
             buf = io.StringIO()
@@ -67,8 +71,20 @@ def test_two_ranks_gloo(tmp_path):
         assert r["max"] == 2.5
         assert r["sum"] == 30.0
         assert r["guard"] == 1.0
-    assert r0["seed"] != r1["seed"]                       # each rank its own batch
-    assert (r0["steps"], r0["img_sum"]) != (r1["steps"], r1["img_sum"])
+    # the two shares are disjoint and together the job's 2 x 8 trajectories
+    assert not set(r0["traj"]) & set(r1["traj"])
+    assert sorted(r0["traj"] + r1["traj"]) == list(range(16))
+    assert r0["steps"] > 0 and r1["steps"] > 0
+    # longest processing time: the busier rank exceeds the mean by at most one trajectory's cost
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2607_11185_gb300 import workloads
+    w = workloads.WORKLOADS["traj8_w3"]
+    gcu, gimg, gtxt = workloads.draw_steps(dataclasses.replace(w, num_traj=16))
+    lens, traj = bench.layout_stats(gcu, gimg, gtxt, w.window, w.keep)
+    per = np.bincount(traj, weights=(lens * (lens + 1) // 2).astype(np.float64), minlength=16)
+    assert r0["cost"] + r1["cost"] == pytest.approx(per.sum())
+    assert max(r0["cost"], r1["cost"]) <= per.sum() / 2 + per.max()
     assert r1["ref_out"] == ""
 
 
@@ -79,11 +95,32 @@ def test_single_process_helpers_are_identity():
     assert not dist.is_initialized()
     assert bench.max_over_ranks(3.25, torch.device("cpu")) == 3.25
     assert bench.sum_over_ranks(7.0, torch.device("cpu")) == 7.0
+    # one rank runs exactly the workload's own draw
     w = workloads.WORKLOADS["traj8_w3"]
-    assert bench.rank_workload(w, 0) is w
-    w1 = bench.rank_workload(w, 1)
-    assert w1.seed != w.seed and (w1.hq, w1.hkv, w1.d, w1.steps, w1.window) == (w.hq, w.hkv, w.d, w.steps, w.window)
+    cu, img, txt, mine = bench.rank_batch(w, w.window, w.keep, 0, 1)
     cu0, img0, txt0 = workloads.draw_steps(w)
-    cu1, img1, txt1 = workloads.draw_steps(w1)
-    assert len(cu0) == len(cu1)                          # same number of trajectories
-    assert not (np.array_equal(cu0, cu1) and np.array_equal(txt0, txt1))
+    assert np.array_equal(cu, cu0) and np.array_equal(img, img0) and np.array_equal(txt, txt0)
+    assert mine == list(range(w.num_traj))
+
+
+def test_lpt_partition():
+    sys.path.insert(0, ROOT)
+    import bench
+    # the textbook case: LPT puts 7 | 6 | 5 first, then 4 on the 5, 3 and 2 on the 6 and 7
+    parts = bench.lpt_partition([7, 6, 5, 4, 3, 2], 3)
+    loads = sorted(sum([7, 6, 5, 4, 3, 2][i] for i in p) for p in parts)
+    assert loads == [9, 9, 9]
+    assert sorted(i for p in parts for i in p) == list(range(6))
+    # equal costs (the long-horizon workload): round robin, equal counts
+    parts = bench.lpt_partition([1.0] * 16, 4)
+    assert [len(p) for p in parts] == [4, 4, 4, 4]
+    # more ranks than units: the extra ranks get nothing
+    assert bench.lpt_partition([5, 1], 3) == [[0], [1], []]
+    # random costs: disjoint cover, and the greedy bound max load <= mean + max cost
+    rng = np.random.default_rng(3)
+    for world in (2, 3, 5, 8):
+        c = rng.integers(1, 1000, 40).astype(float).tolist()
+        parts = bench.lpt_partition(c, world)
+        assert sorted(i for p in parts for i in p) == list(range(40))
+        loads = [sum(c[i] for i in p) for p in parts]
+        assert max(loads) <= sum(c) / world + max(c)
