@@ -35,4 +35,14 @@ def sample_rows(L, rng, n_random=4):
     return sorted(cand)
 
 
+def bench_chunks(w, lay, num_traj):
+    """The chunks the benchmark launches a workload in, as (first segment, end segment) pairs of
+    the oracle's layout: the full-size cases run exactly the launches the benchmark times."""
+    import bench
+    lens = np.diff(np.asarray(lay["cu_seqlens"], np.int64))
+    traj = np.asarray(lay["seg_traj"], np.int64)
+    chunks = bench.make_chunks(lens, traj, num_traj, w.hq, w.hkv, w.d)
+    return [(int(np.searchsorted(traj, b0)), int(np.searchsorted(traj, b1))) for b0, b1 in chunks]
+
+
 WORKLOADS = workloads.WORKLOADS

@@ -12,7 +12,7 @@ import torch
 from oracle import attention as oatt
 from oracle import segments as oseg
 from paper_2607_11185_gb300 import workloads
-from tests.gpu_cases import cu_from_lengths
+from tests.gpu_cases import bench_chunks, cu_from_lengths
 
 pytestmark = pytest.mark.gpu
 
@@ -126,15 +126,16 @@ def check_sampled_grads(q, k, v, do, cu, dq, dk, dv, rng, n_seg=4, n_rows=6, tai
         assert e <= REL, (name, e)
 
 
-def _layout_inputs(name, first_traj=None):
+def _layout_inputs(name, first_chunk=False):
+    """The workload's inputs in segment layout; with first_chunk, only the segments of the
+    benchmark's first launch (its first trajectory chunk)."""
     w = workloads.WORKLOADS[name]
     cu_s, img, txt = workloads.draw_steps(w)
     lay = oseg.build(cu_s, img, txt, w.window, w.keep)
     qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
     cu = lay["cu_seqlens"]
-    if first_traj is not None:
-        ns = int(np.searchsorted(lay["seg_traj"], first_traj))
-        cu = cu[: ns + 1]
+    if first_chunk:
+        cu = cu[: bench_chunks(w, lay, len(cu_s) - 1)[0][1] + 1]
     nt = int(cu[-1])
     g = torch.from_numpy(lay["tok_gather"][:nt].astype(np.int64)).cuda()
     q, k, v = qt[g], kt[g], vt[g]
@@ -149,12 +150,12 @@ def test_traj8_full_size_sampled():
 
 
 def test_traj32_first_chunk_sampled():
-    q, k, v, do, cu = _layout_inputs("traj32_w3", first_traj=8)
+    q, k, v, do, cu = _layout_inputs("traj32_w3", first_chunk=True)
     _, _, dq, dk, dv = run(q, k, v, do, cu)
     check_sampled_grads(q, k, v, do, cu, dq, dk, dv, np.random.default_rng(32), n_seg=2, n_rows=4, tail=16)
 
 
 def test_long_horizon_first_chunk_sampled():
-    q, k, v, do, cu = _layout_inputs("traj16x50_w8", first_traj=4)
+    q, k, v, do, cu = _layout_inputs("traj16x50_w8", first_chunk=True)
     _, _, dq, dk, dv = run(q, k, v, do, cu)
     check_sampled_grads(q, k, v, do, cu, dq, dk, dv, np.random.default_rng(50), n_seg=1, n_rows=3, tail=8)

@@ -13,7 +13,7 @@ import torch
 from oracle import attention as oatt
 from oracle import segments as oseg
 from paper_2607_11185_gb300 import workloads
-from tests.gpu_cases import cu_from_lengths, sample_rows
+from tests.gpu_cases import bench_chunks, cu_from_lengths, sample_rows
 
 pytestmark = pytest.mark.gpu
 
@@ -108,35 +108,35 @@ def check_sampled(q, k, v, cu, o, lse, rng, n_seg=6, heads=None):
     return worst
 
 
-@pytest.mark.parametrize("name", ["traj8_w3", "traj32_w3"])
-def test_workload_full_size_sampled_rows(name):
+def _chunks_sampled(name, seed, **kw):
+    """Every chunk of the workload in the benchmark's launch configuration, on sampled rows."""
     w = workloads.WORKLOADS[name]
     cu_s, img, txt = workloads.draw_steps(w)
     lay = oseg.build(cu_s, img, txt, w.window, w.keep)
     qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
-    g = torch.from_numpy(lay["tok_gather"].astype(np.int64)).cuda()
-    q, k, v = qt[g], kt[g], vt[g]
-    del qt, kt, vt
-    o, lse = run_fwd(q, k, v, lay["cu_seqlens"])
-    check_sampled(q, k, v, lay["cu_seqlens"], o, lse, np.random.default_rng(3))
+    cu = lay["cu_seqlens"]
+    chunks = bench_chunks(w, lay, len(cu_s) - 1)
+    for i, (s0, s1) in enumerate(chunks):
+        t0, t1 = int(cu[s0]), int(cu[s1])
+        g = torch.from_numpy(lay["tok_gather"][t0:t1].astype(np.int64)).cuda()
+        q, k, v = qt[g], kt[g], vt[g]
+        ccu = cu[s0:s1 + 1] - cu[s0]
+        o, lse = run_fwd(q, k, v, ccu)
+        check_sampled(q, k, v, ccu, o, lse, np.random.default_rng(seed + i), **kw)
+        del q, k, v, o, lse
+    return chunks
+
+
+@pytest.mark.parametrize("name", ["traj8_w3", "traj32_w3"])
+def test_workload_full_size_sampled_rows(name):
+    chunks = _chunks_sampled(name, 3)
+    assert len(chunks) == (1 if name == "traj8_w3" else 2)
 
 
 def test_long_horizon_outliers_sampled_rows():
-    # 16 x 50 steps, W=8, 40/8 heads, 5% of K rows scaled by 8; four trajectories at a time
-    w = workloads.WORKLOADS["traj16x50_w8"]
-    cu_s, img, txt = workloads.draw_steps(w)
-    lay = oseg.build(cu_s, img, txt, w.window, w.keep)
-    qt, kt, vt = workloads.draw_traj_qkv(w, workloads.trajectory_tokens(img, txt), device="cuda")
-    cu = lay["cu_seqlens"]
-    # first four trajectories' segments
-    nseg4 = int(np.searchsorted(lay["seg_traj"], 4))
-    ntok4 = int(cu[nseg4])
-    g = torch.from_numpy(lay["tok_gather"][:ntok4].astype(np.int64)).cuda()
-    q, k, v = qt[g], kt[g], vt[g]
-    del qt, kt, vt
-    o, lse = run_fwd(q, k, v, cu[: nseg4 + 1])
-    check_sampled(q, k, v, cu[: nseg4 + 1], o, lse, np.random.default_rng(5),
-                  n_seg=3, heads=[0, 17, 39])
+    # 16 x 50 steps, W=8, 40/8 heads, 5% of K rows scaled by 8; both 8-trajectory chunks
+    chunks = _chunks_sampled("traj16x50_w8", 5, n_seg=3, heads=[0, 17, 39])
+    assert len(chunks) == 2
 
 
 def test_inconsistent_cu_seqlens_reported():
