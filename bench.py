@@ -802,11 +802,14 @@ def run_e2e(path, args, flops, stream):
         avail = int(next(l for l in open("/proc/meminfo") if l.startswith("MemAvailable")).split()[1]) * 1024
     except Exception:
         avail = 0
+    # every rank of this node pins its own copy at the same time, so the node's need is checked;
     # every rank takes the same branch (the decisions are reduced over ranks), so that the
     # collectives below are entered by all of them or by none
-    if sum_over_ranks(float(need > 0.6 * avail), path.dev) > 0:
+    local_ranks = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    if sum_over_ranks(float(need * local_ranks > 0.6 * avail), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s",
-                "error": f"pinned staging of {need / 2**30:.0f} GiB exceeds 60% of available host memory"}
+                "error": f"pinned staging of {local_ranks} x {need / 2**30:.0f} GiB exceeds 60% of available "
+                         f"host memory"}
     host, err = {}, None
     try:
         for name, t in srcs.items():
