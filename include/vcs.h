@@ -381,6 +381,26 @@ vcs_status vcs_grpo_loss(const float* logp, const float* old_logp, const float* 
 vcs_status vcs_group_advantage(const float* rewards, int64_t num_groups, int32_t group_size, float eps, float* adv,
                                void* stream);
 
+/* ------------------------------------------------------------------------ *
+ * Self-test of the bounded device waits.
+ *
+ * The paper has no counterpart to this call.  Every pipeline wait inside the
+ * attention kernels is bounded: a wait that runs out records
+ * VCS_ERR_DEVICE_TIMEOUT in the call's status word, the kernel releases what
+ * it holds and returns, and the CUDA context stays usable.  This call runs the
+ * same mechanism on a barrier that nothing ever arrives on, so a deployment
+ * can check it: one single-thread kernel waits for limit_cycles SM clock
+ * cycles and then writes VCS_ERR_DEVICE_TIMEOUT into *dev_status.
+ *
+ *   dev_status    int32 device word, 4-byte aligned, zeroed by the caller (a
+ *                 nonzero word is left as it is)
+ *   limit_cycles  1 .. 4,000,000,000 (the attention kernels' own limit, about
+ *                 2 s at 2 GHz)
+ * Returns VCS_ERR_INVALID_ARG for a null or misaligned dev_status or a limit
+ * outside that range, before any launch.
+ * ------------------------------------------------------------------------ */
+vcs_status vcs_selftest_bounded_wait(int32_t* dev_status, int64_t limit_cycles, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -77,13 +77,14 @@ _lib_adv = _sig("vcs_group_advantage", _i32, [_p, _i64, _i32, _f32, _p, _p])
 _lib_fields = _sig("vcs_stream_fields", _i32, [_p, _p, _i64, _p, _p, _i64, _p, _p, _p, _p])
 _lib_compact_ws = _sig("vcs_compact_workspace_size", _sz, [_i64])
 _lib_compact = _sig("vcs_compact_trainable", _i32, [_p, _i64, _p, _i64, _p, _p, _sz, _p])
+_lib_selftest_wait = _sig("vcs_selftest_bounded_wait", _i32, [_p, _i64, _p])
 
 EXPORTED = ["vcs_status_string", "vcs_version", "vcs_segments_workspace_size", "vcs_plan_segments",
             "vcs_build_segments", "vcs_gather", "vcs_attn_fwd_workspace_size", "vcs_attn_fwd",
             "vcs_attn_bwd_workspace_size", "vcs_attn_bwd", "vcs_attn_bwd_noalloc", "vcs_grpo_loss_workspace_size",
             "vcs_grpo_loss", "vcs_group_advantage", "vcs_stream_fields", "vcs_compact_workspace_size",
             "vcs_compact_trainable", "vcs_attn_fwd_gathered", "vcs_attn_bwd_gathered_workspace_size",
-            "vcs_attn_bwd_gathered", "vcs_shared_prefix", "vcs_attn_fwd_reuse"]
+            "vcs_attn_bwd_gathered", "vcs_shared_prefix", "vcs_attn_fwd_reuse", "vcs_selftest_bounded_wait"]
 
 LIB_PATH = _LIB_PATH
 
@@ -244,6 +245,10 @@ def vcs_compact_workspace_size(num_tokens: int) -> int:
 def vcs_compact_trainable(tok_loss_mask, num_tokens, idx, idx_capacity, count, ws, ws_bytes, stream=None) -> int:
     return _lib_compact(_ptr(tok_loss_mask), num_tokens, _ptr(idx), idx_capacity, _ptr(count), _ptr(ws), ws_bytes,
                         _stream(stream))
+
+
+def vcs_selftest_bounded_wait(dev_status, limit_cycles, stream=None) -> int:
+    return _lib_selftest_wait(_ptr(dev_status), int(limit_cycles), _stream(stream))
 
 
 # ---------------------------------------------------------------- conveniences
@@ -459,6 +464,16 @@ def group_advantage(rewards, group_size: int, eps: float = 1e-6, stream=None):
     _check(vcs_group_advantage(rewards, rewards.numel() // group_size, group_size, eps, adv, stream),
            "vcs_group_advantage")
     return adv
+
+
+def selftest_bounded_wait(limit_cycles: int = 200_000_000, device="cuda", stream=None) -> int:
+    """Runs the bounded-wait self-test (a wait on a barrier nothing arrives on, given up after
+    limit_cycles SM cycles) and returns the device status it left: VCS_ERR_DEVICE_TIMEOUT (7)
+    when the mechanism works.  Synchronises the device."""
+    status = torch.zeros(1, dtype=torch.int32, device=device)
+    _check(vcs_selftest_bounded_wait(status, limit_cycles, stream), "vcs_selftest_bounded_wait")
+    torch.cuda.synchronize(status.device)
+    return int(status.item())
 
 
 def default_scale(d: int) -> float:

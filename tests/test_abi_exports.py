@@ -97,3 +97,15 @@ def test_gathered_and_reuse_host_checks_without_gpu(lib):
         [ctypes.c_float] + [ctypes.c_void_p] * 3 + [ctypes.c_size_t, ctypes.c_void_p]
     assert fr(A, A, A, A, None, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 4096, None) == 1           # no shared map
     assert fr(A, A, A, A, A, 1, 10, 10, 2, 1, 64, 0.0, A, A, A, 0, None) == 8                 # workspace
+
+
+def test_selftest_bounded_wait_argument_errors_without_gpu(lib):
+    # rejected before any launch: null or misaligned status word, limit outside 1 .. 4e9 cycles
+    f = lib.vcs_selftest_bounded_wait
+    f.restype = ctypes.c_int32
+    f.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p]
+    assert f(None, 1000, None) == 1
+    assert f(258, 1000, None) == 1
+    assert f(256, 0, None) == 1
+    assert f(256, -5, None) == 1
+    assert f(256, 4_000_000_001, None) == 1
