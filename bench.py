@@ -54,16 +54,30 @@ def peaks():
         return 1900.0, 1700.0, 6800.0, "fallback"
 
 
+def backward_code_hash() -> str:
+    """First 16 hex digits of the SHA-256 of the backward's sources (attn_bwd.cu, sm100.cuh) with
+    comments, trailing blanks and blank lines removed: any change to the code changes it, a
+    change to a comment does not."""
+    return code_hash(b"".join(open(os.path.join(ROOT, "paper_2607_11185_gb300", "csrc", f), "rb").read()
+                              for f in ("attn_bwd.cu", "sm100.cuh")))
+
+
+def code_hash(src: bytes) -> str:
+    import hashlib
+    import re
+    src = re.sub(rb"/\*.*?\*/", b"", src, flags=re.S)
+    src = re.sub(rb"//[^\n]*", b"", src)
+    lines = [ln.rstrip() for ln in src.split(b"\n")]
+    return hashlib.sha256(b"\n".join(ln for ln in lines if ln)).hexdigest()[:16]
+
+
 def measured_traffic(profile="attn_bwd_traj16x50_w8.md"):
     """DRAM bytes per vcs_attn_bwd call from the committed ncu capture, or None when the
-    backward kernel sources changed since those counters were taken."""
-    import hashlib
+    backward kernel code changed since those counters were taken."""
     try:
         text = open(os.path.join(ROOT, "profiles", profile)).read()
         vals = dict(line.split(": ", 1) for line in text.splitlines() if ": " in line and " " not in line.split(": ")[0])
-        src = b"".join(open(os.path.join(ROOT, "paper_2607_11185_gb300", "csrc", f), "rb").read()
-                       for f in ("attn_bwd.cu", "sm100.cuh"))
-        if hashlib.sha256(src).hexdigest()[:16] != vals["source_sha256_16"].strip():
+        if backward_code_hash() != vals["code_sha256_16"].strip():
             return None
         return int(vals["traffic_bytes_per_launch"])
     except Exception:

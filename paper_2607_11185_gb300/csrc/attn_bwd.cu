@@ -514,9 +514,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 // compute warpgroups split a tile's query columns.
 //   WG0   warp 0: TMA producer (K and V once, Q/dO 128-row tiles through a 2-stage ring)
 //         warp 1: TMEM allocation and the single MMA-issuing thread
-//   WG1/2 compute, query columns [0,64) / [64,128): S^T, dP^T -> P^T (bf16,
-//         written back to TMEM over dP^T: the A operand of dV += P^T dO) and
-//         dS^T (bf16, shared memory: dK += dS^T Q and dQ = dS K)
+//   WG1/2 compute in two phases, query columns [0,64) then [64,128), warpgroup k
+//         taking 32 columns of each: S^T, dP^T -> P^T (bf16, written back to TMEM
+//         over dP^T: the A operand of dV += P^T dO) and dS^T (bf16, shared memory:
+//         dK += dS^T Q and dQ = dS K); dV and dK over the first phase's columns run
+//         while the second phase is computed
 //   WG3   dQ drain: once a tile's MMAs are complete, dQ (query rows on TMEM
 //         lanes) is copied into the tile's freed Q/dO stage, the columns are
 //         handed back, and TMA bulk reduce-adds add it to the fp32 accumulator

@@ -52,3 +52,10 @@ def test_chunks_cover_the_batch_within_budget(name):
     for a, b in chunks:
         if b - a > 1:                      # a single trajectory may exceed the budget on its own
             assert tok[a:b].sum() * per_tok <= bench.CHUNK_BYTES
+
+
+def test_code_hash_ignores_comments_only():
+    base = b"int a = 1;  // one\n/* block\n comment */ int b = a;\n"
+    assert bench.code_hash(base) == bench.code_hash(b"int a = 1;  // uno\n\n/* other */ int b = a;   \n")
+    assert bench.code_hash(base) != bench.code_hash(b"int a = 2;  // one\n/* block\n comment */ int b = a;\n")
+    assert bench.code_hash(base) != bench.code_hash(b"int a = 1;\nint b = a + 1;\n")
