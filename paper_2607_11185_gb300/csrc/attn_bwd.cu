@@ -389,8 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         dvec_s[buf * 128 + wg * 64 + tw] = next_dd;
       }
       if (it + 1 < iters) load_row_terms(it + 1, next_l2, next_dd);
-      named_bar_sync(1 + wg, 128);
-      if (!mbar_wait(&bars->s_full, it & 1)) { ok = false; break; }
+      // the warpgroup goes on only if every thread finished the previous tile and no role has
+      // given up (a decision all 128 threads take together, so none waits here alone)
+      if (!named_bar_and(1 + wg, 128, ok && !aborted(bars))) { ok = false; break; }
+      // each wait's outcome is the warp's: the TMEM loads that follow are warp-collective
+      if (!mbar_wait_warp(&bars->s_full, it & 1)) { ok = false; continue; }
       tc_fence_after();
       uint32_t sv[64], pv[64];
       tmem_ld_32x32b_x32(trow + C::TM_ST + wg * 64, *reinterpret_cast<uint32_t(*)[32]>(&sv[0]));
@@ -430,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive(&bars->p_full);
       // dQ of this (m, h): query rows on TMEM lanes, this warpgroup's D/2 columns
-      if (!mbar_wait(&bars->dq_full, it & 1)) { ok = false; break; }
+      if (!mbar_wait_warp(&bars->dq_full, it & 1)) { ok = false; continue; }
       tc_fence_after();
       const int qrow = m * C::BN + r;
       float* dst = dq_acc + ((size_t)(start + qrow) * hq + h) * D + wg * (D / 2);
@@ -450,7 +453,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           red_add_v4(dst + e * 4, __uint_as_float(q32[e * 4]), __uint_as_float(q32[e * 4 + 1]),
                      __uint_as_float(q32[e * 4 + 2]), __uint_as_float(q32[e * 4 + 3]));
       }
-      if (aborted(bars)) { ok = false; break; }
     }
     if (!ok) {
       on_timeout(bars, status);
@@ -907,34 +909,39 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       }
       named_bar_sync(1 + k, 128);
       row_terms(u + 1, next_nl2, next_nds);
-      if (!mbar_wait(&bars->s_full, u & 1)) { ok = false; break; }
-      tc_fence_after();
-      // half hf: query columns [64hf + 32k, 64hf + 32k + 32); its P^T (16 words) goes over the
-      // first 16 of its own dP^T columns, its dS^T into chunks 4k..4k+3 of shared block hf
+      // the wait's outcome is the warp's (the TMEM loads below are warp-collective); the
+      // warpgroup decides together at the barrier that closes the tile
+      const bool got = mbar_wait_warp(&bars->s_full, u & 1);
+      if (got) {
+        tc_fence_after();
+        // half hf: query columns [64hf + 32k, 64hf + 32k + 32); its P^T (16 words) goes over the
+        // first 16 of its own dP^T columns, its dS^T into chunks 4k..4k+3 of shared block hf
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        const uint32_t col = 64 * hf + 32 * k;
-        uint32_t sv[32], pv[32], pt[16];
-        tmem_ld_32x32b_x32(trow + C::col_s(u) + col, sv);
-        tmem_ld_32x32b_x32(trow + C::col_p(u) + col, pv);
-        tmem_ld_wait();
-        reg_fence<32>(sv);
-        reg_fence<32>(pv);
-        const uint32_t ds_row = sbase + C::OFF_DS + hf * C::BLOCK + r * 128;
-        if (diag)
-          d128_half_math<true>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, r - (int)col, ds_row, 4 * k, r);
-        else
-          d128_half_math<false>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, 0, ds_row, 4 * k, r);
-        tmem_st_32x32b_x16(trow + C::col_p(u) + col, pt);
-        tmem_st_wait();
-        fence_proxy_async_smem();
-        tc_fence_before();
-        mbar_arrive(&bars->p_full[hf]);
+        for (int hf = 0; hf < 2; ++hf) {
+          const uint32_t col = 64 * hf + 32 * k;
+          uint32_t sv[32], pv[32], pt[16];
+          tmem_ld_32x32b_x32(trow + C::col_s(u) + col, sv);
+          tmem_ld_32x32b_x32(trow + C::col_p(u) + col, pv);
+          tmem_ld_wait();
+          reg_fence<32>(sv);
+          reg_fence<32>(pv);
+          const uint32_t ds_row = sbase + C::OFF_DS + hf * C::BLOCK + r * 128;
+          if (diag)
+            d128_half_math<true>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, r - (int)col, ds_row, 4 * k, r);
+          else
+            d128_half_math<false>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, 0, ds_row, 4 * k, r);
+          tmem_st_32x32b_x16(trow + C::col_p(u) + col, pt);
+          tmem_st_wait();
+          fence_proxy_async_smem();
+          tc_fence_before();
+          mbar_arrive(&bars->p_full[hf]);
+        }
       }
-      named_bar_sync(1 + k, 128);                      // everyone is done with this tile's row terms
-      if (aborted_now()) { ok = false; break; }
+      // everyone is done with this tile's row terms; go on only if every thread got its tile and
+      // no other role has given up
+      if (!named_bar_and(1 + k, 128, got && !aborted_now())) { ok = false; break; }
     }
-    if (ok && !mbar_wait(&bars->acc_done, 0)) ok = false;
+    if (ok) ok = mbar_wait_warp(&bars->acc_done, 0);
     if (!ok) {
       abort_now();
     } else {
@@ -990,27 +997,30 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     bool ok = true;
     for (int u = 0; u < U; ++u) {
       const int stage = u % C::NST;
-      if (!mbar_wait(&bars->kv_done[stage], (u / C::NST) & 1)) { ok = false; break; }
-      tc_fence_after();
+      const bool got = mbar_wait_warp(&bars->kv_done[stage], (u / C::NST) & 1);
       uint8_t* stg = smem + C::OFF_Q + stage * 2 * C::TILE;
-      const uint32_t srow = smem_u32(stg) + l * 128;
+      if (got) {
+        tc_fence_after();
+        const uint32_t srow = smem_u32(stg) + l * 128;
 #pragma unroll
-      for (int part = 0; part < D / 32; ++part) {
-        uint32_t a[32];
-        tmem_ld_32x32b_x32(trow + C::col_s(u) + part * 32, a);
-        tmem_ld_wait();
-        reg_fence<32>(a);
-        if (part == D / 32 - 1) {
-          tc_fence_before();
-          mbar_arrive(&bars->tmem_free);
+        for (int part = 0; part < D / 32; ++part) {
+          uint32_t a[32];
+          tmem_ld_32x32b_x32(trow + C::col_s(u) + part * 32, a);
+          tmem_ld_wait();
+          reg_fence<32>(a);
+          if (part == D / 32 - 1) {
+            tc_fence_before();
+            mbar_arrive(&bars->tmem_free);
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            st_shared_v4(srow + part * (128 * 128) + (uint32_t)((j ^ (l & 7)) << 4), a[4 * j], a[4 * j + 1],
+                         a[4 * j + 2], a[4 * j + 3]);
         }
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          st_shared_v4(srow + part * (128 * 128) + (uint32_t)((j ^ (l & 7)) << 4), a[4 * j], a[4 * j + 1],
-                       a[4 * j + 2], a[4 * j + 3]);
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
-      named_bar_sync(3, 128);
+      // the staged tile is complete, and the warpgroup goes on (or gives up) together
+      if (!named_bar_and(3, 128, got && !aborted_now())) { ok = false; break; }
       if (dw == 0) {
         const int h = head_of(u);
         const int q0 = n * C::BM + sub_of(u) * C::BQ;
@@ -1025,7 +1035,6 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         bulk_wait_read();
         mbar_arrive(&bars->do_free[stage]);
       }
-      if (aborted_now()) { ok = false; break; }
     }
     if (dw == 0) bulk_wait_all();
     if (!ok) abort_now();

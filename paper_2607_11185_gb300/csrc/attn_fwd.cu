@@ -361,8 +361,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_run = -FLT_MAX, l = 0.f;
       bool ok = true;
       for (int j = 0; j <= mt; ++j) {
-        // S(j) complete also means P(j-1) was consumed and O holds P(j-1) V
-        if (!mbar_wait(&bars->s_full[wg], j & 1)) { ok = false; break; }
+        // S(j) complete also means P(j-1) was consumed and O holds P(j-1) V.  The wait's
+        // outcome is the warp's: the TMEM loads and votes below are warp-collective.
+        if (!mbar_wait_warp(&bars->s_full[wg], j & 1)) { ok = false; break; }
         tc_fence_after();
         uint32_t s[128];
 #pragma unroll
@@ -435,9 +436,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&bars->p_full[wg]);
-        if (aborted(bars)) { ok = false; break; }
+        if (__any_sync(0xffffffffu, aborted(bars))) { ok = false; break; }
       }
-      if (ok && !mbar_wait(&bars->o_done[wg], 0)) ok = false;
+      if (ok) ok = mbar_wait_warp(&bars->o_done[wg], 0);
       if (!ok) {
         on_timeout(bars, status);
       } else {
