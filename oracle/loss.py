@@ -22,10 +22,12 @@ no normaliser beyond the expectations; this oracle reads them as follows:
   * group-relative advantage: (r - mean_g r) / (std_g r + eps) over the n
     rollouts of each task, population standard deviation.
 
-Inputs are log-probabilities.  The branch of the clipped objective a token
-takes depends on rho_t; it is decided in the kernel's precision (float32,
-rho = exp(float32(logp - old_logp))) so that both sides take the same branch,
-and the values are then evaluated in fp64.
+Inputs are log-probabilities.  Everything, including the branch of the
+clipped objective a token takes (a comparison of rho_t with 1 - eps_l,
+1 + eps_h and c), is evaluated in fp64 from the given values.  The objective
+is continuous in rho_t, so only the gradient of a token whose ratio lies on a
+branch point depends on the side it is assigned to; there both sides are
+valid sub-gradients.
 """
 from __future__ import annotations
 
@@ -48,12 +50,6 @@ def token_traj(cu_seqlens, seg_traj):
     return np.repeat(st, np.diff(cu))
 
 
-def _branch_rho(logp, old_logp):
-    """rho in the kernel's precision, for the branch decision only."""
-    d = np.asarray(logp, dtype=np.float32) - np.asarray(old_logp, dtype=np.float32)
-    return np.exp(d.astype(np.float32)).astype(np.float32)
-
-
 def grpo_loss(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_traj: int,
               eps_low: float = 0.2, eps_high: float = 0.28, clip_cap: float = 3.0, kl_coef: float = 1e-4):
     """Loss value and its gradient with respect to logp (both fp64).
@@ -67,7 +63,6 @@ def grpo_loss(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_tra
     m = np.asarray(mask).astype(np.float64)
     a = np.asarray(adv, dtype=np.float64)[token_traj(cu_seqlens, seg_traj)]
     n = lp.shape[0]
-    rho32 = _branch_rho(logp, old_logp)
     loss_terms = np.zeros(n)
     grad = np.zeros(n)
     lo, hi = 1.0 - eps_low, 1.0 + eps_high
@@ -76,17 +71,16 @@ def grpo_loss(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num_tra
             continue
         rho = np.exp(lp[t] - old[t])
         A = a[t]
-        rb = float(rho32[t])
         # policy objective o and do/dlogp (rho-dependent branch -> rho*A, constant branch -> 0)
         if A >= 0.0:
-            if rb <= np.float32(hi):
+            if rho <= hi:
                 o, g = rho * A, rho * A
             else:
                 o, g = hi * A, 0.0
         else:
-            if rb < np.float32(lo):
+            if rho < lo:
                 o, g = lo * A, 0.0
-            elif rb > np.float32(clip_cap):
+            elif rho > clip_cap:
                 o, g = clip_cap * A, 0.0
             else:
                 o, g = rho * A, rho * A
@@ -108,12 +102,11 @@ def grpo_loss_vec(logp, old_logp, ref_logp, mask, cu_seqlens, seg_traj, adv, num
     m = np.asarray(mask) != 0
     a = np.asarray(adv, dtype=np.float64)[token_traj(cu_seqlens, seg_traj)]
     rho = np.exp(lp - old)
-    rb = _branch_rho(logp, old_logp)
     lo, hi = 1.0 - eps_low, 1.0 + eps_high
     pos = a >= 0.0
-    const_pos = rb > np.float32(hi)
-    const_lo = rb < np.float32(lo)
-    const_cap = rb > np.float32(clip_cap)
+    const_pos = rho > hi
+    const_lo = rho < lo
+    const_cap = rho > clip_cap
     o = np.where(pos, np.where(const_pos, hi * a, rho * a),
                  np.where(const_lo, lo * a, np.where(const_cap, clip_cap * a, rho * a)))
     dobj = np.where(pos, np.where(const_pos, 0.0, rho * a), np.where(const_lo | const_cap, 0.0, rho * a))
