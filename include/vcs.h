@@ -386,11 +386,12 @@ vcs_status vcs_group_advantage(const float* rewards, int64_t num_groups, int32_t
  *
  * The paper has no counterpart to this call.  Every pipeline wait inside the
  * attention kernels is bounded: a wait that runs out records
- * VCS_ERR_DEVICE_TIMEOUT in the call's status word, the kernel releases what
- * it holds and returns, and the CUDA context stays usable.  This call runs the
- * same mechanism on a barrier that nothing ever arrives on, so a deployment
- * can check it: one single-thread kernel waits for limit_cycles SM clock
- * cycles and then writes VCS_ERR_DEVICE_TIMEOUT into *dev_status.
+ * VCS_ERR_DEVICE_TIMEOUT in the call's status word and the kernel's roles
+ * leave their loops.  This call checks the bounded-wait primitive itself, and
+ * only that: one single-thread kernel waits on a barrier that nothing ever
+ * arrives on for limit_cycles SM clock cycles and then writes
+ * VCS_ERR_DEVICE_TIMEOUT into *dev_status.  How the attention kernels' roles
+ * give up together (warpgroup barriers, TMEM release) is not exercised by it.
  *
  *   dev_status    int32 device word, 4-byte aligned, zeroed by the caller (a
  *                 nonzero word is left as it is)

@@ -134,6 +134,7 @@ static vcs_status check_seg_args(const int32_t* cu_steps, int32_t num_traj, int6
 vcs_status vcs_plan_segments(const int32_t* cu_steps, int32_t num_traj, int64_t num_steps, const int32_t* step_img,
                              const int32_t* step_txt, int32_t window, int32_t keep, vcs_sizes* sizes, void* ws,
                              size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_plan_segments");
   vcs_status s = check_seg_args(cu_steps, num_traj, num_steps, step_img, step_txt, window, keep, sizes, ws, ws_bytes);
   if (s != VCS_OK) return s;
   SegWorkspace w = seg_workspace_carve(ws, num_traj, num_steps);
@@ -148,6 +149,7 @@ vcs_status vcs_build_segments(const int32_t* cu_steps, int32_t num_traj, int64_t
                               int64_t tok_capacity, int32_t* cu_seqlens, int32_t* seg_traj, int32_t* tok_gather,
                               int32_t* tok_src_step, int32_t* tok_pos, uint8_t* tok_loss_mask, vcs_sizes* sizes,
                               void* ws, size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_build_segments");
   vcs_status s = check_seg_args(cu_steps, num_traj, num_steps, step_img, step_txt, window, keep, sizes, ws, ws_bytes);
   if (s != VCS_OK) return s;
   if (seg_capacity < 0 || tok_capacity < 0 || cu_seqlens == nullptr) return VCS_ERR_INVALID_ARG;
@@ -167,6 +169,7 @@ vcs_status vcs_build_segments(const int32_t* cu_steps, int32_t num_traj, int64_t
 vcs_status vcs_gather(const void* q_traj, const void* k_traj, const void* v_traj, int64_t traj_tokens,
                       const int32_t* tok_gather, int64_t num_tokens, int32_t hq, int32_t hkv, int32_t d, void* q,
                       void* k, void* v, int32_t* dev_status, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_gather");
   if (traj_tokens < 0 || num_tokens < 0 || hq <= 0 || d <= 0) return VCS_ERR_INVALID_ARG;
   if (num_tokens > 0 && (tok_gather == nullptr || q_traj == nullptr || q == nullptr)) return VCS_ERR_INVALID_ARG;
   const bool with_kv = k_traj != nullptr || v_traj != nullptr || k != nullptr || v != nullptr;
@@ -219,6 +222,7 @@ size_t vcs_attn_fwd_workspace_size(int32_t num_segments, int64_t num_tokens, int
 vcs_status vcs_attn_fwd(const void* q, const void* k, const void* v, const int32_t* cu_seqlens, int32_t num_segments,
                         int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
                         float softmax_scale, void* o, float* lse, void* ws, size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_fwd");
   AttnArgs a = make_args(q, k, v, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
   vcs_status s = check_attn(a);
   if (s != VCS_OK) return s;
@@ -242,6 +246,7 @@ size_t vcs_attn_bwd_workspace_size(int32_t num_segments, int64_t num_tokens, int
 vcs_status vcs_stream_fields(const int32_t* traj_ids, const float* traj_logp, int64_t traj_tokens,
                              const int32_t* tok_gather, const uint8_t* tok_loss_mask, int64_t num_tokens,
                              int32_t* ids, float* logp, int32_t* dev_status, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_stream_fields");
   if (traj_tokens < 0 || num_tokens < 0) return VCS_ERR_INVALID_ARG;
   if (traj_tokens > INT32_MAX || num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
   if (num_tokens > 0 && (traj_ids == nullptr || traj_logp == nullptr || tok_gather == nullptr ||
@@ -257,6 +262,7 @@ size_t vcs_compact_workspace_size(int64_t num_tokens) { return compact_ws_bytes(
 
 vcs_status vcs_compact_trainable(const uint8_t* tok_loss_mask, int64_t num_tokens, int32_t* idx, int64_t idx_capacity,
                                  int64_t* count, void* ws, size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_compact_trainable");
   if (num_tokens < 0 || idx_capacity < 0 || count == nullptr) return VCS_ERR_INVALID_ARG;
   if (num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
   if (num_tokens > 0 && tok_loss_mask == nullptr) return VCS_ERR_INVALID_ARG;
@@ -277,6 +283,7 @@ vcs_status vcs_grpo_loss(const float* logp, const float* old_logp, const float* 
                          int64_t num_segments, int64_t num_tokens, const float* adv, int64_t num_traj, float eps_low,
                          float eps_high, float clip_cap, float kl_coef, double* loss, float* dlogp, void* ws,
                          size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_grpo_loss");
   if (num_segments < 0 || num_tokens < 0 || num_traj <= 0 || loss == nullptr) return VCS_ERR_INVALID_ARG;
   if (num_tokens > INT32_MAX || num_segments > INT32_MAX || num_traj > INT32_MAX) return VCS_ERR_OVERFLOW;
   if (!(eps_low >= 0.f && eps_low < 1.f) || !(eps_high >= 0.f) || !(clip_cap > 1.f + eps_high) ||
@@ -298,6 +305,7 @@ vcs_status vcs_grpo_loss(const float* logp, const float* old_logp, const float* 
 
 vcs_status vcs_group_advantage(const float* rewards, int64_t num_groups, int32_t group_size, float eps, float* adv,
                                void* stream) {
+  vcs::ApiRange nvtx_range("vcs_group_advantage");
   if (num_groups < 0 || group_size <= 0 || !(eps >= 0.f)) return VCS_ERR_INVALID_ARG;
   if (num_groups > 0 && (rewards == nullptr || adv == nullptr)) return VCS_ERR_INVALID_ARG;
   if (launch_group_advantage(rewards, num_groups, group_size, eps, adv, as_stream(stream)) != cudaSuccess)
@@ -309,6 +317,7 @@ vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void*
                         const void* dout, const int32_t* cu_seqlens, int32_t num_segments, int64_t num_tokens,
                         int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* dq,
                         void* dk, void* dv, void* ws, size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_bwd");
   AttnArgs a = make_args(q, k, v, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
   vcs_status s = check_attn(a);
   if (s != VCS_OK) return s;
@@ -329,6 +338,7 @@ vcs_status vcs_attn_bwd(const void* q, const void* k, const void* v, const void*
 vcs_status vcs_shared_prefix(const int32_t* cu_seqlens, const int32_t* seg_traj, const int32_t* tok_gather,
                              int32_t num_segments, int64_t num_tokens, int32_t* seg_shared, int32_t* dev_status,
                              void* stream) {
+  vcs::ApiRange nvtx_range("vcs_shared_prefix");
   if (num_segments < 0 || num_tokens < 0) return VCS_ERR_INVALID_ARG;
   if (num_tokens > INT32_MAX) return VCS_ERR_OVERFLOW;
   if (num_segments > 0 && (cu_seqlens == nullptr || seg_traj == nullptr || seg_shared == nullptr ||
@@ -344,6 +354,7 @@ vcs_status vcs_attn_fwd_reuse(const void* q, const void* k, const void* v, const
                               const int32_t* seg_shared, int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
                               int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* o, float* lse, void* ws,
                               size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_fwd_reuse");
   AttnArgs a = make_args(q, k, v, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
   vcs_status s = check_attn(a);
   if (s != VCS_OK) return s;
@@ -378,6 +389,7 @@ vcs_status vcs_attn_fwd_gathered(const void* q_traj, const void* k_traj, const v
                                  const int32_t* tok_gather, const int32_t* cu_seqlens, int32_t num_segments,
                                  int64_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d,
                                  float softmax_scale, void* o, float* lse, void* ws, size_t ws_bytes, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_fwd_gathered");
   AttnArgs a =
       make_args(q_traj, k_traj, v_traj, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
   vcs_status s = check_gathered(a, traj_tokens, tok_gather);
@@ -409,6 +421,7 @@ vcs_status vcs_attn_bwd_gathered(const void* q_traj, const void* k_traj, const v
                                  int32_t max_seqlen, int32_t hq, int32_t hkv, int32_t d, float softmax_scale,
                                  void* dq_traj, void* dk_traj, void* dv_traj, void* ws, size_t ws_bytes,
                                  void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_bwd_gathered");
   AttnArgs a =
       make_args(q_traj, k_traj, v_traj, cu_seqlens, num_segments, num_tokens, max_seqlen, hq, hkv, d, softmax_scale);
   vcs_status s = check_gathered(a, traj_tokens, tok_gather);

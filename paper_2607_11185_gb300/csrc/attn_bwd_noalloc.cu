@@ -55,6 +55,7 @@ extern "C" vcs_status vcs_attn_bwd_noalloc(const void* q, const void* k, const v
                                            int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
                                            int32_t hq, int32_t hkv, int32_t d, float softmax_scale, void* dq,
                                            void* dk, void* dv, int32_t* dev_status, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_attn_bwd_noalloc");
   const size_t need = vcs_attn_bwd_workspace_size(num_segments, num_tokens, max_seqlen, hq, hkv, d);
   if (need > vcs::kNoallocScratchBytes) return VCS_ERR_WORKSPACE;
   void* scratch = nullptr;

@@ -6,10 +6,21 @@
 #include <cstddef>
 #include <cstdint>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "vcs.h"
 
 namespace vcs {
+
+// A named NVTX range around one C-ABI call, so that a profiler's timeline (Nsight Systems,
+// Nsight Compute's range filters) shows each entry point and the launches it made.  NVTX is
+// header-only here: with no tool attached a push or pop costs a few nanoseconds.
+struct ApiRange {
+  explicit ApiRange(const char* name) { nvtxRangePushA(name); }
+  ~ApiRange() { nvtxRangePop(); }
+  ApiRange(const ApiRange&) = delete;
+  ApiRange& operator=(const ApiRange&) = delete;
+};
 
 // ---- segment builder (segments.cu) ----
 struct SegWorkspace {

@@ -3,10 +3,10 @@
 //
 // Every pipeline wait in the attention kernels is an mbarrier wait bounded by a
 // cycle limit: when the limit runs out the kernel records VCS_ERR_DEVICE_TIMEOUT
-// in the call's status word, releases its TMEM and returns, and the CUDA context
-// stays usable.  vcs_selftest_bounded_wait runs that mechanism on a barrier that
-// nothing ever arrives on, with a caller-chosen limit, so the host can read the
-// status it leaves.
+// in the call's status word.  vcs_selftest_bounded_wait runs that wait primitive
+// alone, on a barrier that nothing ever arrives on, with a caller-chosen limit,
+// so the host can read the status it leaves.  It does not exercise how a whole
+// attention CTA gives up (its warpgroups' joint decisions, TMEM release).
 #include <cstdint>
 
 #include "internal.h"
@@ -36,6 +36,7 @@ __global__ void __launch_bounds__(1) selftest_wait_kernel(int32_t* status, long 
 }  // namespace vcs
 
 extern "C" vcs_status vcs_selftest_bounded_wait(int32_t* dev_status, int64_t limit_cycles, void* stream) {
+  vcs::ApiRange nvtx_range("vcs_selftest_bounded_wait");
   if (dev_status == nullptr || (reinterpret_cast<uintptr_t>(dev_status) & 3u) != 0) return VCS_ERR_INVALID_ARG;
   if (limit_cycles <= 0 || limit_cycles > vcs::dev::kWaitLimitCycles) return VCS_ERR_INVALID_ARG;
   vcs::selftest_wait_kernel<<<1, 1, 0, static_cast<cudaStream_t>(stream)>>>(dev_status,
