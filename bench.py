@@ -41,7 +41,6 @@ from paper_2607_11185_gb300 import workloads  # noqa: E402
 
 METRIC = "segmented attn fwd+bwd TFLOP/s & % BF16 peak; segment tokens/s; vs CPU oracle"
 CHUNK_BYTES = 130 << 30   # per-chunk working set budget on the device (fewer, larger launches)
-NOMINAL_BF16_TFLOPS = 2250.0  # GB300 dense bf16 tensor rate as NVIDIA quotes it (2:4-sparse figures are 2x)
 
 
 def peaks():
@@ -54,20 +53,29 @@ def peaks():
         return 1900.0, 1700.0, 6800.0, "fallback"
 
 
+BACKWARD_SOURCES = ("attn_bwd.cu", "sm100.cuh", "internal.h", "api.cu")
+
+
 def backward_code_hash() -> str:
-    """First 16 hex digits of the SHA-256 of the backward's sources (attn_bwd.cu, sm100.cuh) with
+    """First 16 hex digits of the SHA-256 of the sources the backward's traffic depends on (its
+    kernels, the PTX wrappers, the workspace layout and argument set-up of the C ABI) with
     comments, trailing blanks and blank lines removed: any change to the code changes it, a
     change to a comment does not."""
     return code_hash(b"".join(open(os.path.join(ROOT, "paper_2607_11185_gb300", "csrc", f), "rb").read()
-                              for f in ("attn_bwd.cu", "sm100.cuh")))
+                              for f in BACKWARD_SOURCES))
+
+
+def strip_comments(src: bytes) -> bytes:
+    """C/C++ source without its comments; string and character literals are kept whole (a
+    '//' inside a string is not a comment)."""
+    import re
+    tok = re.compile(rb'"(?:\\.|[^"\\\n])*"|\'(?:\\.|[^\'\\\n])*\'|/\*.*?\*/|//[^\n]*', re.S)
+    return tok.sub(lambda m: m.group(0) if m.group(0)[:1] in (b'"', b"'") else b"", src)
 
 
 def code_hash(src: bytes) -> str:
     import hashlib
-    import re
-    src = re.sub(rb"/\*.*?\*/", b"", src, flags=re.S)
-    src = re.sub(rb"//[^\n]*", b"", src)
-    lines = [ln.rstrip() for ln in src.split(b"\n")]
+    lines = [ln.rstrip() for ln in strip_comments(src).split(b"\n")]
     return hashlib.sha256(b"\n".join(ln for ln in lines if ln)).hexdigest()[:16]
 
 
@@ -539,7 +547,6 @@ def main():
         "attn_fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "attn_bwd_tflops": f_bwd / (bwd_ms / 1e3) / 1e12,
         "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,
         "frac_of_bf16_burst": value / burst, "frac_of_bf16_sustained": value / sustained,
-        "frac_of_bf16_nominal": value / NOMINAL_BF16_TFLOPS,
         "flash_convention_tflops": value * 14.0 / 12.0,
         "segment_tokens_per_s": job_tokens / (ms / 1e3),
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
@@ -809,9 +816,15 @@ def run_reuse(path, stream, reps=3):
 
 
 def run_e2e(path, args, flops, stream):
-    """Same metric with inputs staged from pinned host memory and results read back."""
+    """Same metric through the public API with host buffers: every step's inputs copied from
+    pinned host memory and every step's result (dQ, dK, dV of every chunk) copied back to
+    pinned host memory, inside the timed region."""
     srcs = {"q": path.q_traj, "k": path.k_traj, "v": path.v_traj, "do": path.dout}
-    need = sum(t.numel() * t.element_size() for t in srcs.values())
+    w = path.w
+    res_shapes = {"dq": (path.num_tokens, w.hq, w.d), "dk": (path.num_tokens, w.hkv, w.d),
+                  "dv": (path.num_tokens, w.hkv, w.d)}
+    need = sum(t.numel() * t.element_size() for t in srcs.values()) + \
+        sum(2 * math.prod(sh) for sh in res_shapes.values())
     try:
         avail = int(next(l for l in open("/proc/meminfo") if l.startswith("MemAvailable")).split()[1]) * 1024
     except Exception:
@@ -823,28 +836,35 @@ def run_e2e(path, args, flops, stream):
     if sum_over_ranks(float(need * local_ranks > 0.6 * avail), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s",
                 "error": f"pinned staging of {local_ranks} x {need / 2**30:.0f} GiB exceeds 60% of available "
-                         f"host memory"}
-    host, err = {}, None
+                         f"host memory ({avail / 2**30:.0f} GiB)"}
+    host, res, err = {}, {}, None
     try:
         for name, t in srcs.items():
             host[name] = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
             host[name].copy_(t)
-        res = torch.empty(path.w.hq * path.max_tok, dtype=torch.float32, pin_memory=True)
+        for name, sh in res_shapes.items():
+            res[name] = torch.empty(sh, dtype=torch.bfloat16, pin_memory=True)
     except RuntimeError as e:
         err = f"pinned staging failed: {e}"[:200]
     if sum_over_ranks(float(err is not None), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s", "error": err or "pinned staging failed on another rank"}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in res.values())
     # Each step's inputs are copied from pinned host memory on a second stream, chunk by
     # chunk: a chunk's copy for the next step starts once its launches of this step are done,
     # so it overlaps the other chunk's compute.  A chunk's builder, gather and forward wait
-    # for its Q/K/V; its backward for its dO (copied after them, under the forward).
+    # for its Q/K/V; its backward for its dO (copied after them, under the forward).  Each
+    # chunk's dQ, dK, dV go back to the host on a third stream as soon as its backward is
+    # done (under the next chunk's builder, gather and forward); the next backward, which
+    # overwrites the device buffers, waits for that copy.
     cs = torch.cuda.Stream(device=path.dev)
+    rs = torch.cuda.Stream(device=path.dev)
     nch = len(path.chunk_in)
     copied = [torch.cuda.Event() for _ in range(nch)]
     copied_do = [torch.cuda.Event() for _ in range(nch)]
     done = [torch.cuda.Event() for _ in range(nch)]
-    state = {"step": 0}
+    returned = [torch.cuda.Event() for _ in range(nch)]
+    state = {"step": 0, "last_return": None}
 
     def copy_chunk(i):
         ci = path.chunk_in[i]
@@ -862,9 +882,20 @@ def run_e2e(path, args, flops, stream):
 
     def before_bwd(i):
         stream.wait_event(copied_do[i])
+        if state["last_return"] is not None:       # the device gradients are still being read
+            stream.wait_event(state["last_return"])
 
     def after(i):
         done[i].record(stream)
+        ci = path.chunk_in[i]
+        n = ci["tok1"] - ci["tok0"]
+        rs.wait_event(done[i])
+        with torch.cuda.stream(rs):
+            res["dq"][ci["tok0"]:ci["tok1"]].copy_(path.dq[:n], non_blocking=True)
+            res["dk"][ci["tok0"]:ci["tok1"]].copy_(path.dk[:n], non_blocking=True)
+            res["dv"][ci["tok0"]:ci["tok1"]].copy_(path.dv[:n], non_blocking=True)
+            returned[i].record(rs)
+        state["last_return"] = returned[i]
         if state["step"] + 1 < args.steps:           # the next step's inputs for this chunk
             cs.wait_event(done[i])
             copy_chunk(i)
@@ -879,14 +910,18 @@ def run_e2e(path, args, flops, stream):
     for s_ in range(args.steps):
         state["step"] = s_
         path.step(stream, before_chunk=before, after_chunk=after, before_bwd=before_bwd)
-        # result read back: the last chunk's log-sum-exp (the loss-side statistic)
-        res.copy_(path.lse.view(-1)[: res.numel()], non_blocking=True)
+    stream.wait_event(state["last_return"])          # the last chunk's gradients are on the host
     t1.record(stream)
     torch.cuda.synchronize()
-    d2h = res.numel() * 4
     ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, path.dev)
+    # the host copy holds the step's gradients: spot-check one row of each against the device
+    ci = path.chunk_in[-1]
+    n = ci["tok1"] - ci["tok0"]
+    for name, dev_t in (("dq", path.dq), ("dk", path.dk), ("dv", path.dv)):
+        assert torch.equal(res[name][ci["tok0"] + n - 1], dev_t[n - 1].cpu()), name
     return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "result": "dQ, dK, dV of every segment token (bf16) copied to pinned host memory every step"}
 
 
 if __name__ == "__main__":

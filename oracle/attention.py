@@ -199,3 +199,45 @@ def keys_dkdv(q, k, v, do, seg, g, keys, scale=None):
             dk[sel] += scale * dsj[:, None] * qi[None, :]
             dv[sel] += p[kj][:, None] * doi[None, :]
     return dk, dv
+
+
+def keys_dkdv_blocked(q, k, v, do, seg, g, keys, scale=None, row_block=512):
+    """dK, dV of kv-head ``g`` for key rows ``keys`` of segment ``seg`` (the same
+    definition as ``keys_dkdv``), with the query rows taken a block at a time.
+
+    A key receives from every later query row of every q-head of its group, and each
+    such row needs its own lse and D = <dO, o>, which depend on all of that row's
+    keys: so every row from min(keys) on is evaluated in full (as in ``attn_fwd``),
+    then its P and dS restricted to the chosen keys are accumulated.  The cost is
+    that of the forward over those rows, which makes keys near the start of long
+    segments reachable.
+    """
+    b, e = seg
+    L = e - b
+    d = q.shape[-1]
+    hq, hkv = q.shape[1], k.shape[1]
+    scale = 1.0 / math.sqrt(d) if scale is None or scale <= 0 else float(scale)
+    keys = np.asarray(keys, dtype=np.int64)
+    kk = _f64(k[b:e, g])
+    vv = _f64(v[b:e, g])
+    dk = np.zeros((len(keys), d))
+    dv = np.zeros((len(keys), d))
+    for h in range(hq):
+        if kv_head(h, hq, hkv) != g:
+            continue
+        qh = _f64(q[b:e, h])
+        doh = _f64(do[b:e, h])
+        for r0 in range(int(keys.min()), L, row_block):
+            r1 = min(L, r0 + row_block)
+            s = _scores(qh, kk, (r0, r1), scale)
+            m = s.max(axis=1)
+            lse = m + np.log(np.exp(s - m[:, None]).sum(axis=1))
+            p = np.exp(s - lse[:, None])
+            dd = (doh[r0:r1] * (p @ vv[:r1])).sum(axis=1)
+            inside = keys < r1                 # later keys are masked for every row of the block
+            kj = keys[inside]
+            pk = p[:, kj]
+            ds = pk * (doh[r0:r1] @ vv[kj].T - dd[:, None])
+            dk[inside] += scale * (ds.T @ qh[r0:r1])
+            dv[inside] += pk.T @ doh[r0:r1]
+    return dk, dv

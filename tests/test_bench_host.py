@@ -59,3 +59,11 @@ def test_code_hash_ignores_comments_only():
     assert bench.code_hash(base) == bench.code_hash(b"int a = 1;  // uno\n\n/* other */ int b = a;   \n")
     assert bench.code_hash(base) != bench.code_hash(b"int a = 2;  // one\n/* block\n comment */ int b = a;\n")
     assert bench.code_hash(base) != bench.code_hash(b"int a = 1;\nint b = a + 1;\n")
+
+
+def test_code_hash_keeps_string_literals():
+    # a '//' or '/*' inside a string literal is code, not a comment
+    a = b'const char* s = "a // b"; int x = 1;\n'
+    b = b'const char* s = "a // c"; int x = 1;\n'
+    assert bench.code_hash(a) != bench.code_hash(b)
+    assert bench.strip_comments(b'f("/* x */"); /* y */ g();') == b'f("/* x */");  g();'

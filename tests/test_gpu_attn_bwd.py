@@ -159,3 +159,48 @@ def test_long_horizon_first_chunk_sampled():
     q, k, v, do, cu = _layout_inputs("traj16x50_w8", first_chunk=True)
     _, _, dq, dk, dv = run(q, k, v, do, cu)
     check_sampled_grads(q, k, v, do, cu, dq, dk, dv, np.random.default_rng(50), n_seg=1, n_rows=3, tail=8)
+
+
+def test_long_horizon_early_and_middle_key_tiles():
+    """dK, dV at full size where the backward does the most work: one kv head of the shortest
+    segment of the benchmark's first long-horizon chunk (L = 25,696), on the first key tile
+    (keys 0-127: every query tile of the segment and all five heads of the group reach it), a
+    tile in the middle of the segment and the ragged last tile, against the oracle evaluated
+    for those keys over all their query rows."""
+    q, k, v, do, cu = _layout_inputs("traj16x50_w8", first_chunk=True)
+    _, _, dq, dk, dv = run(q, k, v, do, cu)
+    lens = np.diff(cu)
+    s = int(np.argmin(lens))
+    b, e = int(cu[s]), int(cu[s + 1])
+    L = e - b
+    mid = (L // 2) // 128 * 128
+    last = (L - 1) // 128 * 128
+    keys = list(range(0, 128)) + list(range(mid, mid + 128)) + list(range(last, L))
+    g = 3
+    rk, rv = oatt.keys_dkdv_blocked(q, k, v, do, (b, e), g, keys, row_block=1024)
+    kidx = torch.tensor([b + j for j in keys], device=dk.device)
+    for name, got, ref in (("dk", dk[kidx, g], rk), ("dv", dv[kidx, g], rv)):
+        got = got.float().cpu().numpy()
+        for lo, hi in ((0, 128), (128, 256), (256, len(keys))):   # each tile on its own
+            err = rel_err(got[lo:hi], ref[lo:hi])
+            assert err <= REL, (name, lo, err)
+
+
+def test_traj8_longest_segment_every_key_and_row():
+    """The 8-trajectory workload's longest segment (5,671 tokens) for one kv head in full: dK,
+    dV of every key and dQ of every row of the group's seven query heads, against the full
+    oracle on that group."""
+    q, k, v, do, cu = _layout_inputs("traj8_w3")
+    _, _, dq, dk, dv = run(q, k, v, do, cu)
+    lens = np.diff(cu)
+    s = int(np.argmax(lens))
+    b, e = int(cu[s]), int(cu[s + 1])
+    hq, hkv = q.shape[1], k.shape[1]
+    G = hq // hkv
+    g = 2
+    heads = slice(g * G, (g + 1) * G)
+    rq, rk, rv = oatt.attn_bwd(q[b:e, heads].cpu(), k[b:e, g:g + 1].cpu(), v[b:e, g:g + 1].cpu(),
+                               do[b:e, heads].cpu(), [0, e - b])
+    for name, got, ref in (("dq", dq[b:e, heads], rq), ("dk", dk[b:e, g:g + 1], rk), ("dv", dv[b:e, g:g + 1], rv)):
+        err = rel_err(got.float().cpu().numpy(), ref)
+        assert err <= REL, (name, err)

@@ -97,7 +97,7 @@ def check_sampled(q, k, v, cu, o, lse, rng, n_seg=6, heads=None):
             continue
         rows = sample_rows(e - b, rng)
         ro, rl = oatt.rows_fwd(q, k, v, (b, e), heads, rows)
-        idx = torch.tensor([b + r for r in rows], device=q.device)
+        idx = torch.tensor([b + r for r in rows], device=o.device)
         got_o = o[idx][:, heads].float().cpu().numpy()
         got_l = lse[heads][:, idx].cpu().numpy()
         eo = np.abs(got_o - ro).max()

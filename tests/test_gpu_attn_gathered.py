@@ -68,6 +68,30 @@ def test_fwd_equals_materialised_gather(name, layout):
     assert torch.equal(lse_g, lse)
 
 
+@pytest.mark.parametrize("name,layout", [("tiny", None), ("traj8_w3", (3, 1))])
+def test_fwd_against_oracle(name, layout):
+    """The gathered forward directly against the fp64 oracle (on the oracle's own gather of the
+    trajectory rows): the tiny workload in full, the 8-trajectory workload with one retained
+    screenshot on sampled rows (O max-abs 2e-2, lse max-abs 2e-3)."""
+    from tests.test_gpu_attn_fwd import LSE_TOL, O_TOL, check_sampled
+    w = workloads.WORKLOADS[name]
+    cu, img, txt = workloads.draw_steps(w)
+    window, keep = layout if layout else (w.window, w.keep)
+    lay, qt, kt, vt, _ = _inputs(cu, img, txt, window, keep, w.hq, w.hkv, w.d, w.seed)
+    vcs = _vcs()
+    o, lse = vcs.attn_fwd_gathered(qt, kt, vt, lay["tok_gather"], lay["cu_seqlens"], lay["max_seqlen"])
+    torch.cuda.synchronize()
+    g = lay["tok_gather"].cpu().numpy()
+    cus = lay["cu_seqlens"].cpu().numpy()
+    q, k, v = og.gather_rows(qt, g), og.gather_rows(kt, g), og.gather_rows(vt, g)
+    if name == "tiny":
+        ro, rl = oatt.attn_fwd(q, k, v, cus)
+        assert np.abs(o.float().cpu().numpy() - ro).max() <= O_TOL
+        assert np.abs(lse.cpu().numpy() - rl).max() <= LSE_TOL
+    else:
+        check_sampled(q, k, v, cus, o, lse, np.random.default_rng(17), n_seg=4)
+
+
 @pytest.mark.parametrize("seed", range(301, 305))
 def test_fwd_random_layouts(seed):
     cu, img, txt = random_steps(seed, max_traj=5, max_T=20, max_img=300, max_txt=40)

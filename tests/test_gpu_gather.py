@@ -62,3 +62,34 @@ def test_gather_out_of_range_index_reported():
     assert st.item() == 6
     assert torch.equal(out[0], q[1]) and torch.equal(out[2], q[3])
     assert torch.all(out[1] == 0) and torch.all(out[3] == 0)
+
+
+def test_gather_long_horizon_chunk_sampled_rows():
+    """The long-horizon workload's first benchmark chunk (40 query / 8 kv heads: 10 KB Q rows,
+    2 KB K and V rows), built and gathered on the GPU from the chunk's own trajectory rows as
+    the benchmark runs it: the chunk's gather map bit-exact against the oracle's, and 4,096
+    sampled rows of Q, K and V (plus the first and last) bit-exact against the oracle's
+    gather."""
+    import dataclasses
+    from paper_2607_11185_gb300 import vcs
+    from tests.gpu_cases import bench_chunks
+    w = workloads.WORKLOADS["traj16x50_w8"]
+    cu, img, txt = workloads.draw_steps(w)
+    lay = oseg.build(cu, img, txt, w.window, w.keep)
+    s0, s1 = bench_chunks(w, lay, len(cu) - 1)[0]
+    b1 = int(lay["seg_traj"][s1 - 1]) + 1                     # the chunk's trajectories: 0 .. b1-1
+    g1 = int(cu[b1])
+    ttok = workloads.trajectory_tokens(img[:g1], txt[:g1])    # its trajectory rows: 0 .. ttok-1
+    t1 = int(lay["cu_seqlens"][s1])
+    glay = vcs.build_segments(*(torch.from_numpy(np.ascontiguousarray(x, np.int32)).cuda()
+                                for x in (cu[:b1 + 1], img[:g1], txt[:g1])), w.window, w.keep)
+    want_map = lay["tok_gather"][:t1]
+    assert np.array_equal(glay["tok_gather"].cpu().numpy(), want_map)
+    q, k, v = workloads.draw_traj_qkv(dataclasses.replace(w, num_traj=b1), ttok, device="cuda")
+    qs, ks, vs = vcs.gather(q, k, v, glay["tok_gather"])
+    rng = np.random.default_rng(55)
+    rows = np.concatenate([[0, t1 - 1], rng.integers(0, t1, size=4096)])
+    rows_t = torch.from_numpy(rows).cuda()
+    for src, got in ((q, qs), (k, ks), (v, vs)):
+        ref = ogather.gather_rows(src.cpu(), want_map[rows])
+        assert torch.equal(got[rows_t].cpu(), ref)

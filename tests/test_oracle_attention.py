@@ -149,3 +149,22 @@ def test_sampled_rows_match_full():
     dk_r, dv_r = att.keys_dkdv(q, k, v, do, seg, 1, keys)
     np.testing.assert_allclose(dk_r, dk[[29 + j for j in keys], 1], atol=1e-12)
     np.testing.assert_allclose(dv_r, dv[[29 + j for j in keys], 1], atol=1e-12)
+
+
+@pytest.mark.parametrize("row_block", [1, 7, 512])
+def test_blocked_key_gradients_match_full(row_block):
+    # the blocked key-gradient function against the full backward and the row-by-row one,
+    # on keys at the start, in the middle and at the end of a ragged segment, GQA 3:1
+    cu = [0, 13, 61]
+    hq, hkv, d = 6, 2, 8
+    q, k, v, do = rand((61, hq, d), 50), rand((61, hkv, d), 51), rand((61, hkv, d), 52), rand((61, hq, d), 53)
+    dq, dk, dv = att.attn_bwd(q, k, v, do, cu)
+    seg = (13, 61)
+    keys = [0, 1, 17, 30, 47]
+    for g in range(hkv):
+        dk_b, dv_b = att.keys_dkdv_blocked(q, k, v, do, seg, g, keys, row_block=row_block)
+        np.testing.assert_allclose(dk_b, dk[[13 + j for j in keys], g], atol=1e-12)
+        np.testing.assert_allclose(dv_b, dv[[13 + j for j in keys], g], atol=1e-12)
+        dk_r, dv_r = att.keys_dkdv(q, k, v, do, seg, g, keys)
+        np.testing.assert_allclose(dk_b, dk_r, atol=1e-12)
+        np.testing.assert_allclose(dv_b, dv_r, atol=1e-12)

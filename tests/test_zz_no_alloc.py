@@ -5,14 +5,16 @@ owns all device memory and passes it only the input and output tensors, or a
 latency-critical loop that must not call cudaMalloc.  vcs_attn_bwd_noalloc
 serves them from a fixed scratch array inside the library.  These tests call
 it through the C ABI and check it against vcs_attn_bwd (the entry point with
-a caller workspace) on two calls in a row, which share the same scratch, and
-check that a problem larger than the scratch is refused before any launch.
+a caller workspace) and against the fp64 oracle on two calls in a row, which
+share the same scratch, and check that a problem larger than the scratch is
+refused before any launch.
 This file runs last so that a failure here leaves every other test run.
 """
 import numpy as np
 import pytest
 import torch
 
+from oracle import attention as oatt
 from paper_2607_11185_gb300 import workloads
 from tests.gpu_cases import cu_from_lengths
 
@@ -47,6 +49,10 @@ def test_noalloc_matches_workspace_entry_point_twice(d):
         assert status.item() == 0
         for got, want in zip((dq, dk, dv), ref):
             assert rel(got, want) <= REL
+        # and directly against the oracle, so that a fault shared by both entry points shows
+        exact = oatt.attn_bwd(q.cpu(), k.cpu(), v.cpu(), do.cpu(), cu)
+        for got, want in zip((dq, dk, dv), exact):
+            assert rel(got.cpu(), torch.from_numpy(want)) <= REL
 
 
 def test_noalloc_refuses_problems_larger_than_its_scratch():
