@@ -823,16 +823,23 @@ def run_e2e(path, args, flops, stream):
     w = path.w
     res_shapes = {"dq": (path.num_tokens, w.hq, w.d), "dk": (path.num_tokens, w.hkv, w.d),
                   "dv": (path.num_tokens, w.hkv, w.d)}
-    need = sum(t.numel() * t.element_size() for t in srcs.values()) + \
-        sum(2 * math.prod(sh) for sh in res_shapes.values())
+    need_in = sum(t.numel() * t.element_size() for t in srcs.values())
     try:
         avail = int(next(l for l in open("/proc/meminfo") if l.startswith("MemAvailable")).split()[1]) * 1024
     except Exception:
         avail = 0
     # every rank of this node pins its own copy at the same time, so the node's need is checked;
     # every rank takes the same branch (the decisions are reduced over ranks), so that the
-    # collectives below are entered by all of them or by none
+    # collectives below are entered by all of them or by none.  The result buffers hold the
+    # whole step's gradients when they fit beside the inputs; otherwise one chunk's, which every
+    # chunk's gradients pass through in turn (the bytes copied back per step are the same).
     local_ranks = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    res_rows = path.num_tokens
+    if sum_over_ranks(float((need_in + sum(2 * math.prod(sh) for sh in res_shapes.values())) * local_ranks
+                            > 0.6 * avail), path.dev) > 0:
+        res_rows = path.max_tok
+        res_shapes = {k: (res_rows,) + sh[1:] for k, sh in res_shapes.items()}
+    need = need_in + sum(2 * math.prod(sh) for sh in res_shapes.values())
     if sum_over_ranks(float(need * local_ranks > 0.6 * avail), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s",
                 "error": f"pinned staging of {local_ranks} x {need / 2**30:.0f} GiB exceeds 60% of available "
@@ -849,7 +856,8 @@ def run_e2e(path, args, flops, stream):
     if sum_over_ranks(float(err is not None), path.dev) > 0:
         return {"value": None, "unit": "TFLOP/s", "error": err or "pinned staging failed on another rank"}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = sum(t.numel() * t.element_size() for t in res.values())
+    d2h = path.num_tokens * (w.hq + 2 * w.hkv) * w.d * 2          # every chunk's dQ, dK, dV
+    whole = res_rows == path.num_tokens
     # Each step's inputs are copied from pinned host memory on a second stream, chunk by
     # chunk: a chunk's copy for the next step starts once its launches of this step are done,
     # so it overlaps the other chunk's compute.  A chunk's builder, gather and forward wait
@@ -890,10 +898,11 @@ def run_e2e(path, args, flops, stream):
         ci = path.chunk_in[i]
         n = ci["tok1"] - ci["tok0"]
         rs.wait_event(done[i])
+        r0 = ci["tok0"] if whole else 0              # copies on rs run in order: a shared buffer is free
         with torch.cuda.stream(rs):
-            res["dq"][ci["tok0"]:ci["tok1"]].copy_(path.dq[:n], non_blocking=True)
-            res["dk"][ci["tok0"]:ci["tok1"]].copy_(path.dk[:n], non_blocking=True)
-            res["dv"][ci["tok0"]:ci["tok1"]].copy_(path.dv[:n], non_blocking=True)
+            res["dq"][r0:r0 + n].copy_(path.dq[:n], non_blocking=True)
+            res["dk"][r0:r0 + n].copy_(path.dk[:n], non_blocking=True)
+            res["dv"][r0:r0 + n].copy_(path.dv[:n], non_blocking=True)
             returned[i].record(rs)
         state["last_return"] = returned[i]
         if state["step"] + 1 < args.steps:           # the next step's inputs for this chunk
@@ -917,11 +926,15 @@ def run_e2e(path, args, flops, stream):
     # the host copy holds the step's gradients: spot-check one row of each against the device
     ci = path.chunk_in[-1]
     n = ci["tok1"] - ci["tok0"]
+    r0 = ci["tok0"] if whole else 0
     for name, dev_t in (("dq", path.dq), ("dk", path.dk), ("dv", path.dv)):
-        assert torch.equal(res[name][ci["tok0"] + n - 1], dev_t[n - 1].cpu()), name
+        assert torch.equal(res[name][r0 + n - 1], dev_t[n - 1].cpu()), name
     return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "result": "dQ, dK, dV of every segment token (bf16) copied to pinned host memory every step"}
+            "result": "dQ, dK, dV of every segment token (bf16) copied to pinned host memory every step, into "
+                      + ("buffers holding the whole step" if whole else
+                         "one chunk-sized buffer per tensor that each chunk's gradients pass through (the whole "
+                         "step's would not fit beside the pinned inputs in 60% of the host's available memory)")}
 
 
 if __name__ == "__main__":
