@@ -548,21 +548,35 @@ __device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.w
 __device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-// One compute thread's share of a half tile: key row r against 32 query columns.
+// TMEM loads / stores of N consecutive 32-bit columns of the warp's 32 lanes.
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&r)[N]) {
+  static_assert(N == 16 || N == 32, "16 or 32 columns");
+  if constexpr (N == 32) tmem_ld_32x32b_x32(taddr, r);
+  else tmem_ld_32x32b_x16(taddr, r);
+}
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)[N]) {
+  static_assert(N == 8 || N == 16, "8 or 16 columns");
+  if constexpr (N == 16) tmem_st_32x32b_x16(taddr, r);
+  else tmem_st_32x32b_x8(taddr, r);
+}
+
+// One compute thread's share of one phase: key row r against NC query columns.
 //   P^T  = 2^(S^T * scale*log2e - lse*log2e)     (zero where the key follows the query)
 //   dS^T = P^T * (dP^T - D) * scale
 // The row terms come as {-lse*log2e, -D*scale} of each column pair, one 16-byte load
 // {nl(c), nl(c+1), nd(c), nd(c+1)} per pair.  P^T goes to pt as bf16 pairs; dS^T to
-// 16-byte chunks CH0 .. CH0+3 of the thread's 128-byte row of the swizzled K-major
+// 16-byte chunks CH0 .. CH0+NC/8-1 of the thread's 128-byte row of the swizzled K-major
 // shared block.  The causal test is compiled
 // only into the diagonal instantiation (column c is masked when c < dlim), so the
 // off-diagonal tiles run a branch-free body the compiler can interleave.
-template <bool DIAG>
-__device__ __forceinline__ void d128_half_math(const uint32_t (&sv)[32], const uint32_t (&pv)[32], uint32_t (&pt)[16],
-                                               const float* rt, uint64_t sl2, uint64_t sc2, int dlim, uint32_t ds_row,
-                                               int ch0, int r) {
+template <int NC, bool DIAG>
+__device__ __forceinline__ void d128_phase_math(const uint32_t (&sv)[NC], const uint32_t (&pv)[NC],
+                                                uint32_t (&pt)[NC / 2], const float* rt, uint64_t sl2, uint64_t sc2,
+                                                int dlim, uint32_t ds_row, int ch0, int r) {
 #pragma unroll
-  for (int ch = 0; ch < 4; ++ch) {
+  for (int ch = 0; ch < NC / 8; ++ch) {
     uint32_t wd[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -591,6 +605,13 @@ struct D128 {
   static constexpr int BM = 128;                 // key rows of the tile
   static constexpr int BQ = 128;                 // query rows per tile
   static constexpr int NST = 2;                  // Q/dO ring stages
+  // The compute runs in NPH phases of PW query columns; warpgroup k takes columns
+  // [PW*ph + HW*k, PW*ph + HW*k + HW) of phase ph, and dV, dK over a phase's columns are
+  // issued as soon as both warpgroups have written them.
+  static constexpr int NPH = 4;
+  static constexpr int PW = 128 / NPH;
+  static constexpr int HW = PW / 2;
+  static constexpr int KPP = PW / 16;            // K = 16 MMA steps (16 queries each) per phase
   static constexpr int THREADS = 512;
   static constexpr int TILE = 128 * D * 2;       // 32 KB: K, V, a Q or a dO tile
   static constexpr int BLOCK = 128 * 128;        // one 64-column block of a 128-row tile
@@ -605,6 +626,11 @@ struct D128 {
   // tile u: S^T (later dQ) in TM_A for even u, TM_B for odd u; dP^T (later P^T) in the other
   __device__ static uint32_t col_s(int u) { return (u & 1) ? TM_B : TM_A; }
   __device__ static uint32_t col_p(int u) { return (u & 1) ? TM_A : TM_B; }
+  // P^T of queries [16kk, 16kk+16) (8 columns of bf16 pairs) is written by the warpgroup that
+  // computes them, into the first columns of the dP^T columns it has itself just read
+  __host__ __device__ static constexpr uint32_t pt_col(int kk) {
+    return PW * (kk / KPP) + HW * ((kk % KPP) / (KPP / 2)) + 8 * (kk % (KPP / 2));
+  }
   static constexpr int REG_CTRL = 104, REG_COMPUTE = 176, REG_DRAIN = 56;
   static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
@@ -623,7 +649,7 @@ struct D128Bars {
   uint64_t q_free[D128::NST];      // the drain's reduce-adds have read the stage's Q half
   uint64_t do_free[D128::NST];     // ... and its dO half
   uint64_t s_full;
-  uint64_t p_full[2];  // query columns [0,64) / [64,128) of the tile: P^T and dS^T written
+  uint64_t p_full[D128::NPH];  // the query columns of phase ph of the tile: P^T and dS^T written
   uint64_t tmem_free;
   uint64_t acc_done;
   uint32_t tmem_base;
@@ -689,8 +715,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       mbar_init(&bars->do_free[i], 1);
     }
     mbar_init(&bars->s_full, 1);
-    mbar_init(&bars->p_full[0], 256);
-    mbar_init(&bars->p_full[1], 256);
+    for (int i = 0; i < C::NPH; ++i) mbar_init(&bars->p_full[i], 256);
     mbar_init(&bars->tmem_free, 128);
     mbar_init(&bars->acc_done, 1);
     bars->abort = 0;
@@ -836,29 +861,32 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           tc_mma_ss(cp, desc_at(v_kmaj, o), desc_at(dd, o), C::IDESC_S, kk > 0);
         }
         tc_commit(&bars->s_full);
-        // dV += P^T dO and dK += dS^T Q over the first 64 queries as soon as they are
-        // written (overlapping the compute of the other 64), then dQ = dS K and the rest
-        // of dV, dK.  In-order execution keeps S(u+1) from overwriting P^T or dS^T first.
-        // P^T of queries [16kk, 16kk+16) sits at column 64(kk/4) + 32((kk/2)%2) + 8(kk%2).
+        // dV += P^T dO and dK += dS^T Q over each phase's queries as soon as they are written
+        // (overlapping the compute of the next phase), then, after the last phase, dQ = dS K
+        // and the last phase's dV, dK.  In-order execution keeps S(u+1) from overwriting P^T or
+        // dS^T first.  P^T of queries [16kk, 16kk+16) sits at C::pt_col(kk) of its columns.
         const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::TILE), dmn = desc_at(qmn, C::TILE);
         const uint32_t acc0 = u > 0 ? 1u : 0u;
         auto issue_dvdk = [&](int kk0) {
 #pragma unroll
-          for (int kk = kk0; kk < kk0 + 4; ++kk)
-            tc_mma_ts(tmem + C::TM_DV, cp + (kk >> 2) * 64 + ((kk >> 1) & 1) * 32 + (kk & 1) * 8,
-                      desc_at(dmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+          for (int kk = kk0; kk < kk0 + C::KPP; ++kk)
+            tc_mma_ts(tmem + C::TM_DV, cp + C::pt_col(kk), desc_at(dmn, kk * 2048), C::IDESC_KV,
+                      kk > 0 ? 1u : acc0);
 #pragma unroll
-          for (int kk = kk0; kk < kk0 + 4; ++kk)
+          for (int kk = kk0; kk < kk0 + C::KPP; ++kk)
             tc_mma_ss(tmem + C::TM_DK, desc_at(ds_kmaj, (kk >> 2) * C::BLOCK + (kk & 3) * 32),
                       desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
         };
-        if (!mbar_wait(&bars->p_full[0], u & 1)) {
-          ok = false;
-          break;
+#pragma unroll
+        for (int ph = 0; ph < C::NPH - 1; ++ph) {
+          if (!mbar_wait(&bars->p_full[ph], u & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_dvdk(ph * C::KPP);
         }
-        tc_fence_after();
-        issue_dvdk(0);
-        if (!mbar_wait(&bars->p_full[1], u & 1)) {
+        if (!ok || !mbar_wait(&bars->p_full[C::NPH - 1], u & 1)) {
           ok = false;
           break;
         }
@@ -867,7 +895,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         for (int kk = 0; kk < C::BM / 16; ++kk)
           tc_mma_ss(cs, desc_at(ds_mnmaj, kk * 2048), desc_at(k_mnmaj, kk * 2048), C::IDESC_DQ,
                     kk > 0 ? 1u : 0u);
-        issue_dvdk(4);
+        issue_dvdk((C::NPH - 1) * C::KPP);
         tc_commit(&bars->kv_done[stage]);
       }
       tc_commit(&bars->acc_done);
@@ -884,14 +912,16 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     // row terms of the warpgroup's 64 query columns, per half of 32: {nl(c), nl(c+1), nd(c), nd(c+1)}
     // for each column pair, nl = -lse*log2e and nd = -D*scale
     float* rt_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;
-    const int rt_slot = (tw >> 5) * 64 + ((tw & 31) >> 1) * 4 + (tw & 1);  // this thread's column (tw < 64)
+    // thread tw < 64 stages the terms of column HW*k + PW*(tw / HW) + tw % HW; phase ph's terms
+    // start at rt_s + PW*ph
+    const int rt_slot = (tw / C::HW) * C::PW + ((tw % C::HW) >> 1) * 4 + (tw & 1);
     const uint64_t sl2 = f2pack(scale_log2, scale_log2), sc2 = f2pack(scale, scale);
     auto row_terms = [&](int u, float& nl2, float& nds) {
       nl2 = __int_as_float(0xff800000);  // -inf: query outside the segment -> P = 0
       nds = 0.f;
       if (u < U && tw < 64) {
         const int h = head_of(u);
-        const int q = n * C::BM + sub_of(u) * C::BQ + (tw < 32 ? 32 * k + tw : 32 + 32 * k + tw);
+        const int q = n * C::BM + sub_of(u) * C::BQ + C::PW * (tw / C::HW) + C::HW * k + tw % C::HW;
         if (q < L) {
           nl2 = -__ldg(&lse[(size_t)h * num_tokens + start + q]) * 1.4426950408889634f;
           nds = -__ldg(&dvec[(size_t)h * num_tokens + start + q]) * scale;
@@ -914,27 +944,29 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const bool got = mbar_wait_warp(&bars->s_full, u & 1);
       if (got) {
         tc_fence_after();
-        // half hf: query columns [64hf + 32k, 64hf + 32k + 32); its P^T (16 words) goes over the
-        // first 16 of its own dP^T columns, its dS^T into chunks 4k..4k+3 of shared block hf
+        // phase ph: query columns [PW*ph + HW*k, PW*ph + HW*k + HW); its P^T (HW/2 words) goes
+        // over the first of its own dP^T columns, its dS^T into HW/8 16-byte chunks of the
+        // shared block of its 64 queries
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-          const uint32_t col = 64 * hf + 32 * k;
-          uint32_t sv[32], pv[32], pt[16];
-          tmem_ld_32x32b_x32(trow + C::col_s(u) + col, sv);
-          tmem_ld_32x32b_x32(trow + C::col_p(u) + col, pv);
+        for (int ph = 0; ph < C::NPH; ++ph) {
+          const uint32_t col = C::PW * ph + C::HW * k;
+          uint32_t sv[C::HW], pv[C::HW], pt[C::HW / 2];
+          tmem_ld_cols<C::HW>(trow + C::col_s(u) + col, sv);
+          tmem_ld_cols<C::HW>(trow + C::col_p(u) + col, pv);
           tmem_ld_wait();
-          reg_fence<32>(sv);
-          reg_fence<32>(pv);
-          const uint32_t ds_row = sbase + C::OFF_DS + hf * C::BLOCK + r * 128;
+          reg_fence<C::HW>(sv);
+          reg_fence<C::HW>(pv);
+          const uint32_t ds_row = sbase + C::OFF_DS + (col / 64) * C::BLOCK + r * 128;
+          const int ch0 = (int)(col % 64) / 8;
           if (diag)
-            d128_half_math<true>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, r - (int)col, ds_row, 4 * k, r);
+            d128_phase_math<C::HW, true>(sv, pv, pt, rt_s + C::PW * ph, sl2, sc2, r - (int)col, ds_row, ch0, r);
           else
-            d128_half_math<false>(sv, pv, pt, rt_s + 64 * hf, sl2, sc2, 0, ds_row, 4 * k, r);
-          tmem_st_32x32b_x16(trow + C::col_p(u) + col, pt);
+            d128_phase_math<C::HW, false>(sv, pv, pt, rt_s + C::PW * ph, sl2, sc2, 0, ds_row, ch0, r);
+          tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col, pt);
           tmem_st_wait();
           fence_proxy_async_smem();
           tc_fence_before();
-          mbar_arrive(&bars->p_full[hf]);
+          mbar_arrive(&bars->p_full[ph]);
         }
       }
       // everyone is done with this tile's row terms; go on only if every thread got its tile and
