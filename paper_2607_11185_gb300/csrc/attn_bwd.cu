@@ -573,15 +573,16 @@ __device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)
 // off-diagonal tiles run a branch-free body the compiler can interleave.
 template <int NC, bool DIAG>
 __device__ __forceinline__ void d128_phase_math(const uint32_t (&sv)[NC], const uint32_t (&pv)[NC],
-                                                uint32_t (&pt)[NC / 2], const float* rt, uint64_t sl2, uint64_t sc2,
-                                                int dlim, uint32_t ds_row, int ch0, int r) {
+                                                uint32_t (&pt)[NC / 2], const uint4 (&rq)[NC / 2], uint64_t sl2,
+                                                uint64_t sc2, int dlim, uint32_t ds_row, int ch0, int r) {
 #pragma unroll
   for (int ch = 0; ch < NC / 8; ++ch) {
     uint32_t wd[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int c = ch * 8 + e * 2;
-      const float4 q = *reinterpret_cast<const float4*>(&rt[2 * c]);
+      const float4 q = make_float4(__uint_as_float(rq[c / 2].x), __uint_as_float(rq[c / 2].y),
+                                   __uint_as_float(rq[c / 2].z), __uint_as_float(rq[c / 2].w));
       float x0, x1;
       f2unpack(ffma2(f2pack(__uint_as_float(sv[c]), __uint_as_float(sv[c + 1])), sl2, f2pack(q.x, q.y)), x0, x1);
       float p0 = ex2(x0), p1 = ex2(x1);
@@ -912,6 +913,7 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     // row terms of the warpgroup's 64 query columns, per half of 32: {nl(c), nl(c+1), nd(c), nd(c+1)}
     // for each column pair, nl = -lse*log2e and nd = -D*scale
     float* rt_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;
+    const uint32_t rt_u32 = smem_u32(rt_s);
     // thread tw < 64 stages the terms of column HW*k + PW*(tw / HW) + tw % HW; phase ph's terms
     // start at rt_s + PW*ph
     const int rt_slot = (tw / C::HW) * C::PW + ((tw % C::HW) >> 1) * 4 + (tw & 1);
@@ -947,26 +949,43 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         // phase ph: query columns [PW*ph + HW*k, PW*ph + HW*k + HW); its P^T (HW/2 words) goes
         // over the first of its own dP^T columns, its dS^T into HW/8 16-byte chunks of the
         // shared block of its 64 queries
+        // the next phase's S^T and dP^T columns are loaded while this phase is computed
+        uint32_t sv[2][C::HW], pv[2][C::HW];
+        tmem_ld_cols<C::HW>(trow + C::col_s(u) + C::HW * k, sv[0]);
+        tmem_ld_cols<C::HW>(trow + C::col_p(u) + C::HW * k, pv[0]);
+        tmem_ld_wait();
+        reg_fence<C::HW>(sv[0]);
+        reg_fence<C::HW>(pv[0]);
 #pragma unroll
         for (int ph = 0; ph < C::NPH; ++ph) {
+          const int cur = ph & 1;
           const uint32_t col = C::PW * ph + C::HW * k;
-          uint32_t sv[C::HW], pv[C::HW], pt[C::HW / 2];
-          tmem_ld_cols<C::HW>(trow + C::col_s(u) + col, sv);
-          tmem_ld_cols<C::HW>(trow + C::col_p(u) + col, pv);
-          tmem_ld_wait();
-          reg_fence<C::HW>(sv);
-          reg_fence<C::HW>(pv);
+          if (ph + 1 < C::NPH) {
+            tmem_ld_cols<C::HW>(trow + C::col_s(u) + col + C::PW, sv[cur ^ 1]);
+            tmem_ld_cols<C::HW>(trow + C::col_p(u) + col + C::PW, pv[cur ^ 1]);
+          }
+          // the phase's row terms, all loads issued back to back so that their latencies overlap
+          uint4 rq[C::HW / 2];
+#pragma unroll
+          for (int e = 0; e < C::HW / 2; ++e) rq[e] = ld_shared_v4(rt_u32 + (uint32_t)(C::PW * ph + 4 * e) * 4);
+          uint32_t pt[C::HW / 2];
           const uint32_t ds_row = sbase + C::OFF_DS + (col / 64) * C::BLOCK + r * 128;
           const int ch0 = (int)(col % 64) / 8;
           if (diag)
-            d128_phase_math<C::HW, true>(sv, pv, pt, rt_s + C::PW * ph, sl2, sc2, r - (int)col, ds_row, ch0, r);
+            d128_phase_math<C::HW, true>(sv[cur], pv[cur], pt, rq, sl2, sc2, r - (int)col, ds_row, ch0, r);
           else
-            d128_phase_math<C::HW, false>(sv, pv, pt, rt_s + C::PW * ph, sl2, sc2, 0, ds_row, ch0, r);
+            d128_phase_math<C::HW, false>(sv[cur], pv[cur], pt, rq, sl2, sc2, 0, ds_row, ch0, r);
+          // dS^T (shared memory) is published to the tensor pipe while P^T's TMEM store completes
+          fence_proxy_async_smem();
           tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col, pt);
           tmem_st_wait();
-          fence_proxy_async_smem();
           tc_fence_before();
           mbar_arrive(&bars->p_full[ph]);
+          if (ph + 1 < C::NPH) {
+            tmem_ld_wait();
+            reg_fence<C::HW>(sv[cur ^ 1]);
+            reg_fence<C::HW>(pv[cur ^ 1]);
+          }
         }
       }
       // everyone is done with this tile's row terms; go on only if every thread got its tile and
