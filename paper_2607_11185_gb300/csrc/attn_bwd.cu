@@ -524,7 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 //   WG3   dQ drain: once a tile's MMAs are complete, dQ (query rows on TMEM
 //         lanes) is copied into the tile's freed Q/dO stage, the columns are
 //         handed back, and TMA bulk reduce-adds add it to the fp32 accumulator
-// Registers are rebalanced per warpgroup with setmaxnreg (104 / 176 / 176 / 56
+// Registers are rebalanced per warpgroup with setmaxnreg (96 / 168 / 168 / 80
 // per thread; the block launches with 128).
 // With a 64-query sub-tile and two streams (compute of one stream overlapping
 // the other's MMAs) the N = 64 MMAs held the backward 5% lower on the
@@ -632,7 +632,7 @@ struct D128 {
   __host__ __device__ static constexpr uint32_t pt_col(int kk) {
     return PW * (kk / KPP) + HW * ((kk % KPP) / (KPP / 2)) + 8 * (kk % (KPP / 2));
   }
-  static constexpr int REG_CTRL = 104, REG_COMPUTE = 176, REG_DRAIN = 56;
+  static constexpr int REG_CTRL = 96, REG_COMPUTE = 168, REG_DRAIN = 80;
   static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
   static constexpr uint32_t IDESC_KV = idesc_bf16(128, 128, 0, 1);  // P^T (TMEM) / dS^T (K-major) x dO / Q (MN-major)
@@ -1053,20 +1053,26 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       if (got) {
         tc_fence_after();
         const uint32_t srow = smem_u32(stg) + l * 128;
+        // two 32-column parts per TMEM round trip, so that the columns are handed back after two
+        // rounds of loads
 #pragma unroll
-        for (int part = 0; part < D / 32; ++part) {
-          uint32_t a[32];
-          tmem_ld_32x32b_x32(trow + C::col_s(u) + part * 32, a);
+        for (int pp = 0; pp < D / 64; ++pp) {
+          uint32_t a[2][32];
+          tmem_ld_32x32b_x32(trow + C::col_s(u) + pp * 64, a[0]);
+          tmem_ld_32x32b_x32(trow + C::col_s(u) + pp * 64 + 32, a[1]);
           tmem_ld_wait();
-          reg_fence<32>(a);
-          if (part == D / 32 - 1) {
+          reg_fence<32>(a[0]);
+          reg_fence<32>(a[1]);
+          if (pp == D / 64 - 1) {
             tc_fence_before();
             mbar_arrive(&bars->tmem_free);
           }
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            st_shared_v4(srow + part * (128 * 128) + (uint32_t)((j ^ (l & 7)) << 4), a[4 * j], a[4 * j + 1],
-                         a[4 * j + 2], a[4 * j + 3]);
+          for (int i = 0; i < 2; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              st_shared_v4(srow + (2 * pp + i) * (128 * 128) + (uint32_t)((j ^ (l & 7)) << 4), a[i][4 * j],
+                           a[i][4 * j + 1], a[i][4 * j + 2], a[i][4 * j + 3]);
         }
         fence_proxy_async_smem();
       }
