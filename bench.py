@@ -79,15 +79,17 @@ def code_hash(src: bytes) -> str:
     return hashlib.sha256(b"\n".join(ln for ln in lines if ln)).hexdigest()[:16]
 
 
-def measured_traffic(profile="attn_bwd_traj16x50_w8.md"):
-    """DRAM bytes per vcs_attn_bwd call from the committed ncu capture, or None when the
-    backward kernel code changed since those counters were taken."""
+def measured_traffic(trajectories, profile="attn_traffic_traj16x50_w8_1traj.md"):
+    """DRAM bytes per vcs_attn_bwd call of `trajectories` long-horizon trajectories, from the
+    committed ncu capture of a one-trajectory small case (every trajectory of that workload has the
+    same segments, so the bytes scale with the trajectory count), or None when the backward's code
+    changed since those counters were taken."""
     try:
         text = open(os.path.join(ROOT, "profiles", profile)).read()
         vals = dict(line.split(": ", 1) for line in text.splitlines() if ": " in line and " " not in line.split(": ")[0])
         if backward_code_hash() != vals["code_sha256_16"].strip():
             return None
-        return int(vals["traffic_bytes_per_launch"])
+        return int(vals["traffic_bytes_per_trajectory"]) * int(trajectories)
     except Exception:
         return None
 
@@ -450,11 +452,17 @@ def main():
     ap.add_argument("--no-fused", action="store_true", help="skip the gathered-attention (fused gather) timing")
     ap.add_argument("--no-reuse", action="store_true", help="skip the prefix-reuse forward timing")
     ap.add_argument("--no-hbm-kernels", action="store_true", help="skip the builder / gather timings")
+    ap.add_argument("--num-traj", type=int, default=None,
+                    help="run the first NUM_TRAJ trajectories of the workload's draw instead of all (a small case "
+                         "of the same segment shapes, for profiler captures); the line's config says so")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     w = workloads.WORKLOADS[args.workload]
+    if args.num_traj is not None:
+        import dataclasses
+        w = dataclasses.replace(w, num_traj=args.num_traj)
     window, keep = w.window, w.keep
     if args.layout is not None:
         window, keep = workloads.COMPARISON_LAYOUTS[args.layout]
@@ -552,8 +560,10 @@ def main():
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
                      "achieved": ach_bwd, "peak": sustained, "unit": "TFLOP/s", "frac": ach_bwd / sustained,
                      "peak_source": f"{src} bf16 sustained",
-                     "traffic": measured_traffic() if w.name == "traj16x50_w8" and (window, keep) == (w.window, w.keep)
-                     else None},
+                     "traffic": measured_traffic(path.chunk_in[0]["b1"] - path.chunk_in[0]["b0"])
+                     if w.name == "traj16x50_w8" and (window, keep) == (w.window, w.keep) else None,
+                     "traffic_source": "ncu DRAM bytes of a one-trajectory small case x the trajectories of a "
+                                       "launch (profiles/attn_traffic_traj16x50_w8_1traj.md)"},
         "cpu_baseline": cpu,
         "e2e": e2e,
         "next_rows": next_rows,
