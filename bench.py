@@ -234,9 +234,10 @@ class Path:
         self.bwd_ws = T(self.bwd_ws_bytes, dt=torch.uint8)
         self.launches_per_step = 0
 
-    def step(self, tstream, ev=None, before_chunk=None, after_chunk=None, before_bwd=None):
+    def step(self, tstream, ev=None, before_chunk=None, after_chunk=None, before_bwd=None, grads=None):
         """One pass of the hot path over all chunks; optional per-chunk events appended to ev and
-        hooks called before a chunk's first launch, before its backward and after its last one."""
+        hooks called before a chunk's first launch, before its backward and after its last one;
+        grads(i) gives chunk i's (dq, dk, dv) output buffers (default: the path's own)."""
         vcs, w = self.vcs, self.w
         stream = tstream.cuda_stream
         hq, hkv, d = w.hq, w.hkv, w.d
@@ -279,9 +280,10 @@ class Path:
             dout = self.dout[ci["tok0"]:ci["tok1"]]
             if before_bwd is not None:
                 before_bwd(i)
+            dq, dk, dv = (self.dq, self.dk, self.dv) if grads is None else grads(i)
             st = vcs.vcs_attn_bwd(self.q, self.k, self.v, self.o, self.lse, dout, self.cu_seqlens, nseg, ntok,
-                                  ci["max_seqlen"], hq, hkv, d, 0.0, self.dq, self.dk, self.dv, self.bwd_ws,
-                                  self.bwd_ws_bytes, stream)
+                                  ci["max_seqlen"], hq, hkv, d, 0.0, dq, dk, dv, self.bwd_ws, self.bwd_ws_bytes,
+                                  stream)
             launches += 3
             assert st == 0
             if evs:
@@ -452,6 +454,8 @@ def main():
     ap.add_argument("--no-fused", action="store_true", help="skip the gathered-attention (fused gather) timing")
     ap.add_argument("--no-reuse", action="store_true", help="skip the prefix-reuse forward timing")
     ap.add_argument("--no-hbm-kernels", action="store_true", help="skip the builder / gather timings")
+    ap.add_argument("--builder-stress-traj", type=int, default=4096,
+                    help="trajectories of the builder stress batch (a smaller one for profiler captures)")
     ap.add_argument("--num-traj", type=int, default=None,
                     help="run the first NUM_TRAJ trajectories of the workload's draw instead of all (a small case "
                          "of the same segment shapes, for profiler captures); the line's config says so")
@@ -535,7 +539,7 @@ def main():
     next_rows = None if args.no_next_rows else run_next_rows(path, stream, hbm)
     fused = None if args.no_fused else run_fused(path, stream)
     reuse = None if args.no_reuse else run_reuse(path, stream)
-    hbm_kernels = None if args.no_hbm_kernels else run_hbm_kernels(path, stream, hbm)
+    hbm_kernels = None if args.no_hbm_kernels else run_hbm_kernels(path, stream, hbm, args.builder_stress_traj)
 
     ach_bwd = bwd_launch_flops / (bwd_launch_ms / 1e3) / 1e12
     line = {
@@ -878,11 +882,15 @@ def run_e2e(path, args, flops, stream):
     cs = torch.cuda.Stream(device=path.dev)
     rs = torch.cuda.Stream(device=path.dev)
     nch = len(path.chunk_in)
+    # chunks alternate between two sets of device gradient buffers, so that a chunk's backward
+    # never waits for the previous chunk's gradients to reach the host
+    gsets = [(path.dq, path.dk, path.dv), tuple(torch.empty_like(t) for t in (path.dq, path.dk, path.dv))]
+    chunk_no = {"n": 0}
+    set_of = {}
     copied = [torch.cuda.Event() for _ in range(nch)]
     copied_do = [torch.cuda.Event() for _ in range(nch)]
     done = [torch.cuda.Event() for _ in range(nch)]
-    returned = [torch.cuda.Event() for _ in range(nch)]
-    state = {"step": 0, "last_return": None}
+    state = {"step": 0, "returned": [None, None]}
 
     def copy_chunk(i):
         ci = path.chunk_in[i]
@@ -898,23 +906,32 @@ def run_e2e(path, args, flops, stream):
     def before(i):
         stream.wait_event(copied[i])
 
+    def grads(i):
+        k = chunk_no["n"] % 2                        # this chunk's gradient buffer set
+        set_of[i] = k
+        chunk_no["n"] += 1
+        return gsets[k]
+
     def before_bwd(i):
         stream.wait_event(copied_do[i])
-        if state["last_return"] is not None:       # the device gradients are still being read
-            stream.wait_event(state["last_return"])
+        k = chunk_no["n"] % 2
+        if state["returned"][k] is not None:        # that set's last gradients are still being read
+            stream.wait_event(state["returned"][k])
 
     def after(i):
         done[i].record(stream)
         ci = path.chunk_in[i]
         n = ci["tok1"] - ci["tok0"]
+        k = set_of[i]
         rs.wait_event(done[i])
         r0 = ci["tok0"] if whole else 0              # copies on rs run in order: a shared buffer is free
         with torch.cuda.stream(rs):
-            res["dq"][r0:r0 + n].copy_(path.dq[:n], non_blocking=True)
-            res["dk"][r0:r0 + n].copy_(path.dk[:n], non_blocking=True)
-            res["dv"][r0:r0 + n].copy_(path.dv[:n], non_blocking=True)
-            returned[i].record(rs)
-        state["last_return"] = returned[i]
+            for name, t in zip(("dq", "dk", "dv"), gsets[k]):
+                res[name][r0:r0 + n].copy_(t[:n], non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(rs)
+        state["returned"][k] = ev
+        state["last"] = (ev, k)
         if state["step"] + 1 < args.steps:           # the next step's inputs for this chunk
             cs.wait_event(done[i])
             copy_chunk(i)
@@ -928,8 +945,8 @@ def run_e2e(path, args, flops, stream):
         copy_chunk(i)
     for s_ in range(args.steps):
         state["step"] = s_
-        path.step(stream, before_chunk=before, after_chunk=after, before_bwd=before_bwd)
-    stream.wait_event(state["last_return"])          # the last chunk's gradients are on the host
+        path.step(stream, before_chunk=before, after_chunk=after, before_bwd=before_bwd, grads=grads)
+    stream.wait_event(state["last"][0])              # the last chunk's gradients are on the host
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, path.dev)
@@ -937,7 +954,7 @@ def run_e2e(path, args, flops, stream):
     ci = path.chunk_in[-1]
     n = ci["tok1"] - ci["tok0"]
     r0 = ci["tok0"] if whole else 0
-    for name, dev_t in (("dq", path.dq), ("dk", path.dk), ("dv", path.dv)):
+    for name, dev_t in zip(("dq", "dk", "dv"), gsets[state["last"][1]]):
         assert torch.equal(res[name][r0 + n - 1], dev_t[n - 1].cpu()), name
     return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
