@@ -679,7 +679,6 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   D128Bars* bars = reinterpret_cast<D128Bars*>(smem + C::OFF_BAR);
 
-  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
   const int sg = (int)(blockIdx.z * 65535u + blockIdx.y);
   if (sg >= num_segments * hkv) return;
   const int seg = sg / hkv;
@@ -694,6 +693,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
   }
   const int L = end - start;
   if (n * C::BM >= L) return;
+  // once any CTA of this launch has given up on a wait, the rest stand down (read only by the
+  // CTAs that have a key tile)
+  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
   const int G = hq / hkv;
   const int nsub = (L - n * C::BM + C::BQ - 1) / C::BQ;  // 128-row query tiles at or after this key tile
   const int U = G * nsub;

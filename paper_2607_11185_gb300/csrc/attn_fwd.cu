@@ -153,8 +153,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
-  // once any CTA of this launch has given up on a wait, the rest stand down
-  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
   // 1-D grid ordered (segment, kv-head, pair from the last, head in group):
   // the CTAs that stream the same K/V tiles are launched together, so those
   // tiles are read from HBM about once and then served from L2
@@ -176,6 +174,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   const int L = end - start;
   if (p * 2 * C::BM >= L) return;  // this pair of query tiles lies beyond the segment
+  // once any CTA of this launch has given up on a wait, the rest stand down (read only by the
+  // CTAs that have work: the grid is sized by the longest segment, and most of a short
+  // segment's CTAs leave above after their two cu_seqlens loads)
+  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
   // prefix reuse: the pair's rows equal the previous segment's (copied by fwd_reuse_copy)
   if (seg_shared != nullptr && (p + 1) * 2 * C::BM <= reuse_skip_rows(seg_shared, cu_seqlens, seg, status)) return;
   const int m0 = 2 * p, m1 = 2 * p + 1;
