@@ -419,6 +419,20 @@ def sum_over_ranks(value: float, device) -> float:
     return float(t.item())
 
 
+def line_config(w, window, keep, cu, img, txt, world):
+    """The workload a line was measured on (the same for both arms): sizes of the layout this rank
+    runs, from the closed form on the host."""
+    seg_lens, seg_traj = layout_stats(cu, img, txt, window, keep)
+    chunks = make_chunks(seg_lens, seg_traj, len(cu) - 1, w.hq, w.hkv, w.d)
+    return {"workload": w.name, "window": window, "keep": keep, "num_traj": w.num_traj, "hq": w.hq, "hkv": w.hkv,
+            "d": w.d, "segments": int(len(seg_lens)), "segment_tokens": int(seg_lens.sum()),
+            "max_seqlen": int(seg_lens.max()) if len(seg_lens) else 0, "chunks": len(chunks),
+            "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)",
+            **({"sharding": f"{world * w.num_traj} trajectories over {world} ranks by longest processing "
+                            f"time on sum L(L+1)/2; segments, tokens and chunks above are rank 0's"}
+               if world > 1 else {})}
+
+
 def run_reference(args, w, window, keep, rank, world):
     if rank != 0:
         return
@@ -433,7 +447,7 @@ def run_reference(args, w, window, keep, rank, world):
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": secs * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "window": window, "keep": keep, "hq": w.hq, "hkv": w.hkv, "d": w.d},
+            "config": line_config(w, window, keep, *rank_batch(w, window, keep, rank, world)[:3], world),
             "cpu_baseline": cpu,
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -546,13 +560,7 @@ def main():
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": w.name, "window": window, "keep": keep, "num_traj": w.num_traj, "hq": w.hq,
-                   "hkv": w.hkv, "d": w.d, "segments": int(len(path.seg_lens)), "segment_tokens": path.num_tokens,
-                   "max_seqlen": int(path.seg_lens.max()), "chunks": len(path.chunk_in),
-                   "l2": "inputs larger than L2 (trajectory Q/K/V and dO resident, > 129 MB)",
-                   **({"sharding": f"{world * w.num_traj} trajectories over {world} ranks by longest processing "
-                                   f"time on sum L(L+1)/2; segments, tokens and chunks above are rank 0's"}
-                      if world > 1 else {})},
+        "config": line_config(w, window, keep, path.cu, path.img, path.txt, world),
         "attn_tflop_credited": flops / 1e12,
         "builder_ms": build_ms, "gather_ms": gather_ms, "gather_gbs": gather_bytes / (gather_ms / 1e3) / 1e9,
         "attn_fwd_ms": fwd_ms, "attn_bwd_ms": bwd_ms,
