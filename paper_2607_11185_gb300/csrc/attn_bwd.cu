@@ -516,14 +516,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 // compute warpgroups split a tile's query columns.
 //   WG0   warp 0: TMA producer (K and V once, Q/dO 128-row tiles through a 2-stage ring)
 //         warp 1: TMEM allocation and the single MMA-issuing thread
-//   WG1/2 compute in two phases, query columns [0,64) then [64,128), warpgroup k
-//         taking 32 columns of each: S^T, dP^T -> P^T (bf16, written back to TMEM
-//         over dP^T: the A operand of dV += P^T dO) and dS^T (bf16, shared memory:
-//         dK += dS^T Q and dQ = dS K); dV and dK over the first phase's columns run
-//         while the second phase is computed
+//   WG1/2 compute in four phases of 32 query columns, warpgroup k taking 16
+//         columns of each: S^T, dP^T -> P^T (bf16, written back to TMEM over the
+//         warpgroup's own dP^T columns: the A operand of dV += P^T dO) and dS^T
+//         (bf16, shared memory: dK += dS^T Q and dQ = dS K); dV and dK over a
+//         phase's columns run while the next phase is computed
 //   WG3   dQ drain: once a tile's MMAs are complete, dQ (query rows on TMEM
-//         lanes) is copied into the tile's freed Q/dO stage, the columns are
-//         handed back, and TMA bulk reduce-adds add it to the fp32 accumulator
+//         lanes) is read two 32-column parts at a time and copied into the tile's
+//         freed Q/dO stage, the columns are handed back, and TMA bulk reduce-adds
+//         add it to the fp32 accumulator
 // Registers are rebalanced per warpgroup with setmaxnreg (96 / 168 / 168 / 80
 // per thread; the block launches with 128).
 // With a 64-query sub-tile and two streams (compute of one stream overlapping
@@ -912,7 +913,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     const int r = quad * 32 + lane;  // TMEM lane: key row
     const int tw = threadIdx.x - 128 - k * 128;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
-    // row terms of the warpgroup's 64 query columns, per half of 32: {nl(c), nl(c+1), nd(c), nd(c+1)}
+    // row terms of the warpgroup's 64 query columns, per phase (16 columns):
+    // {nl(c), nl(c+1), nd(c), nd(c+1)}
     // for each column pair, nl = -lse*log2e and nd = -D*scale
     float* rt_s = reinterpret_cast<float*>(smem + C::OFF_ROW) + k * 128;
     const uint32_t rt_u32 = smem_u32(rt_s);
