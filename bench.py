@@ -221,6 +221,10 @@ class Path:
         self.tok_pos = T(max_tok, dt=torch.int32)
         self.tok_mask = T(max_tok, dt=torch.uint8)
         self.sizes = torch.zeros(3, dtype=torch.int64, device=device)
+        # each chunk's builder writes its layout sizes to a slot of its own, read back and checked
+        # against the host's closed form once the timed steps are done (verify_sizes): the step
+        # itself never waits for the device
+        self.sizes_all = torch.zeros((len(self.chunks), 3), dtype=torch.int64, device=device)
         self.seg_ws_bytes = vcs.vcs_segments_workspace_size(max(b1 - b0 for b0, b1 in self.chunks), max_steps)
         self.seg_ws = T(self.seg_ws_bytes, dt=torch.uint8)
         self.q, self.k, self.v = T(max_tok, hq, d), T(max_tok, hkv, d), T(max_tok, hkv, d)
@@ -251,15 +255,15 @@ class Path:
                 evs[0].record(tstream)
             st = vcs.vcs_build_segments(ci["cu"], ci["b1"] - ci["b0"], ci["nsteps"], ci["img"], ci["txt"],
                                         self.window, self.keep, self.max_seg, self.max_tok, self.cu_seqlens, None,
-                                        self.tok_gather, self.tok_src, self.tok_pos, self.tok_mask, self.sizes,
-                                        self.seg_ws, self.seg_ws_bytes, stream)
+                                        self.tok_gather, self.tok_src, self.tok_pos, self.tok_mask,
+                                        self.sizes_all[i], self.seg_ws, self.seg_ws_bytes, stream)
             launches += 5
             assert st == 0, vcs.vcs_status_string(st)
             if evs:
                 evs[1].record(tstream)
-            # the attention launch shape depends on the layout sizes: read them (one sync per chunk)
-            sz = self.sizes.cpu()
-            assert int(sz[0]) == nseg and int(sz[1]) == ntok and (int(sz[2]) >> 32) == 0
+            # the attention launches take the layout sizes the host computed from the closed form
+            # (the trajectories' step counts are the host's own input); the builder's sizes are
+            # checked against them after the timed steps (verify_sizes)
             qt = self.q_traj[ci["ttok0"]:ci["ttok1"]]
             kt = self.k_traj[ci["ttok0"]:ci["ttok1"]]
             vt = self.v_traj[ci["ttok0"]:ci["ttok1"]]
@@ -292,6 +296,13 @@ class Path:
             if after_chunk is not None:
                 after_chunk(i)
         self.launches_per_step = launches
+
+    def verify_sizes(self):
+        """The builder's layout sizes of every chunk (from the last step) equal the host's."""
+        sz = self.sizes_all.cpu()
+        for i, ci in enumerate(self.chunk_in):
+            assert int(sz[i, 0]) == ci["s1"] - ci["s0"] and int(sz[i, 1]) == ci["tok1"] - ci["tok0"], (i, sz[i])
+            assert int(sz[i, 2]) & 0xffffffff == ci["max_seqlen"] and (int(sz[i, 2]) >> 32) == 0, (i, sz[i])
 
     def device_status(self):
         return (int(self.gstatus.item()), int(self.fwd_ws[:4].view(torch.int32).item()),
@@ -510,6 +521,7 @@ def main():
     torch.cuda.synchronize()
     st = path.device_status()
     assert st == (0, 0, 0), f"device status {st}"
+    path.verify_sizes()
 
     def barrier():
         if world > 1:
@@ -528,6 +540,7 @@ def main():
     t1.record(stream)
     barrier()
     ck = clocks.stop()
+    path.verify_sizes()
     ms = t0.elapsed_time(t1) / args.steps
     ms = max_over_ranks(ms, dev)
     # per chunk: [0]-[1] build, (host reads the sizes), [2]-[3] gather, [3]-[4] fwd, [4]-[5] bwd
@@ -958,6 +971,7 @@ def run_e2e(path, args, flops, stream):
     t1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, path.dev)
+    path.verify_sizes()
     # the host copy holds the step's gradients: spot-check one row of each against the device
     ci = path.chunk_in[-1]
     n = ci["tok1"] - ci["tok0"]
