@@ -149,6 +149,12 @@ vcs_status vcs_gather(const void* q_traj, const void* k_traj, const void* v_traj
  * for a wait that gave up); every call clears it first.
  * ------------------------------------------------------------------------ */
 
+/* Forward workspace: the header, then the list of the launch's work units (one
+ * per segment, query head and pair of 128-row query tiles, 16 bytes each, at
+ * most hq * (num_tokens / 256 + num_segments + 1) of them) and their
+ * per-segment offsets, built on the device by the call itself; about
+ * hq * num_tokens / 16 bytes.  Also the size for vcs_attn_fwd_reuse and
+ * vcs_attn_fwd_gathered. */
 size_t vcs_attn_fwd_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
                                    int32_t hq, int32_t hkv, int32_t d);
 

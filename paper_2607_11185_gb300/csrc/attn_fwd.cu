@@ -10,10 +10,18 @@
 // 128-row query tiles (m0 = 2p, m1 = 2p+1).  Both tiles stream the same K/V
 // tiles of kv-head h / (hq/hkv), so each K/V tile brought into shared memory
 // feeds 256 query rows.  Tiles above the diagonal are never visited; only the
-// diagonal tile is masked element-wise.  Grid: one dimension ordered by
-// (segment, kv-head, pair index from the last, query head in the group), so
-// the CTAs sharing a K/V stream run together and the longest pairs of each
-// stream start first.
+// diagonal tile is masked element-wise.
+//
+// Grid: two small kernels first list the launch's work units in device memory
+// (fwd_item_scan counts each segment's pairs and checks the segment bounds,
+// fwd_item_fill writes {start, end, pair, head} per unit), in the order
+// (segment, kv-head, pair index from the last, query head in the group); CTA
+// b takes unit b.  The CTAs sharing a K/V stream run together, so those tiles
+// are read from HBM about once and then served from L2, and the longest pairs
+// of each stream start first.  Pairs beyond a segment's end are not listed
+// (a grid sized by the longest segment would launch them only to exit), and
+// neither are pairs that prefix reuse copies from the previous segment; the
+// grid is an upper bound of the count, and the few CTAs past it exit at once.
 //
 // Warp roles (384 threads):
 //   warp 0      TMA producer: Q0/Q1 once, then K and V tiles into a 5-slot ring
@@ -86,6 +94,9 @@ struct Bars {
   int32_t abort;
 };
 
+// workspace header: the number of listed work units sits after the status word
+constexpr size_t kWsItemTotal = 128;
+
 __device__ __forceinline__ void on_timeout(Bars* b, int32_t* status) {
   set_status(status, VCS_ERR_DEVICE_TIMEOUT);
   *reinterpret_cast<volatile int32_t*>(&b->abort) = 1;
@@ -132,6 +143,89 @@ __device__ __forceinline__ int reuse_skip_rows(const int32_t* __restrict__ seg_s
   return sh / 256 * 256;
 }
 
+// Pairs of query tiles of segment s the forward computes: none for a segment whose bounds are
+// invalid (recorded as a device check), and none of those that prefix reuse copies from the
+// previous segment.  Pairs [np - count, np) remain, np = ceil(L / 256).
+__device__ __forceinline__ int seg_item_pairs(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
+                                              int32_t num_tokens, int32_t max_seqlen,
+                                              const int32_t* __restrict__ seg_shared, int s, int32_t* status) {
+  const int start = cu_seqlens[s], end = cu_seqlens[s + 1];
+  if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen || (s == 0 && start != 0) ||
+      (s == num_segments - 1 && end != num_tokens)) {
+    set_status(status, VCS_ERR_DEVICE_CHECK);
+    return 0;
+  }
+  const int np = (end - start + 255) / 256;
+  return np - reuse_skip_rows(seg_shared, cu_seqlens, s, status) / 256;
+}
+
+// off[s] = hq * (pairs of segments 0 .. s-1), off[S] = *total: one block, in chunks of 1024
+// segments (warp scans, then a scan of the warp sums).
+__global__ void __launch_bounds__(1024) fwd_item_scan(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
+                                                      int32_t num_tokens, int32_t max_seqlen, int32_t hq,
+                                                      const int32_t* __restrict__ seg_shared,
+                                                      int32_t* __restrict__ off, int32_t* __restrict__ total,
+                                                      int32_t* status) {
+  __shared__ int32_t wsum[32];
+  __shared__ int32_t carry;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < num_segments; base += 1024) {
+    const int s = base + (int)threadIdx.x;
+    const int cnt =
+        s < num_segments ? hq * seg_item_pairs(cu_seqlens, num_segments, num_tokens, max_seqlen, seg_shared, s, status)
+                         : 0;
+    int x = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) wsum[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+      int w = wsum[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += y;
+      }
+      wsum[lane] = w;
+    }
+    __syncthreads();
+    const int incl = carry + (wid > 0 ? wsum[wid - 1] : 0) + x;
+    if (s < num_segments) off[s] = incl - cnt;
+    __syncthreads();
+    if (threadIdx.x == 1023) carry = incl;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    off[num_segments] = carry;
+    *total = carry;
+  }
+}
+
+// The units of segment s at off[s] .. off[s+1]-1, in the order (kv head, pair from the last,
+// query head in the group): {segment start, segment end, pair index, query head}.
+__global__ void __launch_bounds__(256) fwd_item_fill(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
+                                                     int32_t hq, int32_t hkv, const int32_t* __restrict__ off,
+                                                     int4* __restrict__ items) {
+  const int G = hq / hkv;
+  for (int s = blockIdx.x; s < num_segments; s += gridDim.x) {
+    const int base = off[s], n = off[s + 1] - base;
+    if (n == 0) continue;
+    const int start = cu_seqlens[s], end = cu_seqlens[s + 1];
+    const int np = (end - start + 255) / 256;
+    const int cnt = n / hq;  // pairs np - cnt .. np - 1
+    for (int r = threadIdx.x; r < n; r += blockDim.x) {
+      const int hh = r % G, r2 = r / G;
+      const int pr = r2 % cnt, g = r2 / cnt;
+      items[base + r] = make_int4(start, end, np - 1 - pr, g * G + hh);
+    }
+  }
+}
+
 // GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
 // tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr and
 // tm_qs/ks/vs 3-D tiled maps of the same tensors (128- and 32-row boxes) for tiles or
@@ -140,12 +234,12 @@ __device__ __forceinline__ int reuse_skip_rows(const int32_t* __restrict__ seg_s
 template <int D, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v, const int32_t* __restrict__ cu_seqlens,
-                    int32_t num_segments, int32_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv,
-                    int32_t npairs, float scale_log2, __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
+                    const __grid_constant__ CUtensorMap tm_v, const int4* __restrict__ items,
+                    const int32_t* __restrict__ item_total, int32_t num_tokens, int32_t hq, int32_t hkv,
+                    float scale_log2, __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
                     int32_t* status, const int32_t* __restrict__ tok_gather, int32_t traj_tokens,
                     const __grid_constant__ CUtensorMap tm_qr, const __grid_constant__ CUtensorMap tm_kr,
-                    const __grid_constant__ CUtensorMap tm_vr, const int32_t* __restrict__ seg_shared,
+                    const __grid_constant__ CUtensorMap tm_vr,
                     const __grid_constant__ CUtensorMap tm_qs, const __grid_constant__ CUtensorMap tm_ks,
                     const __grid_constant__ CUtensorMap tm_vs) {
   using C = Fwd<D>;
@@ -153,33 +247,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   Bars* bars = reinterpret_cast<Bars*>(smem + C::OFF_BAR);
 
-  // 1-D grid ordered (segment, kv-head, pair from the last, head in group):
-  // the CTAs that stream the same K/V tiles are launched together, so those
-  // tiles are read from HBM about once and then served from L2
+  // CTA b takes listed unit b; the unit, the count and the status word are loaded together
   const int G = hq / hkv;
-  int idx = (int)blockIdx.x;
-  const int hh = idx % G;
-  idx /= G;
-  const int p = npairs - 1 - idx % npairs;
-  idx /= npairs;
-  const int g = idx % hkv;
-  const int seg = idx / hkv;
-  const int h = g * G + hh;
-  const int start = cu_seqlens[seg];
-  const int end = cu_seqlens[seg + 1];
-  if (start < 0 || end < start || end > num_tokens || end - start > max_seqlen ||
-      (seg == 0 && start != 0) || (seg == num_segments - 1 && end != num_tokens)) {
-    if (threadIdx.x == 0 && p == 0 && h == 0) set_status(status, VCS_ERR_DEVICE_CHECK);
-    return;
-  }
+  const int4 e = items[blockIdx.x];
+  const int total = *item_total;
+  const int st = *reinterpret_cast<volatile int32_t*>(status);
+  if ((int)blockIdx.x >= total) return;  // the grid is an upper bound of the listed units
+  // once any CTA of this launch has given up on a wait, the rest stand down
+  if (st == VCS_ERR_DEVICE_TIMEOUT) return;
+  const int start = e.x, end = e.y, p = e.z, h = e.w, g = h / G;
   const int L = end - start;
-  if (p * 2 * C::BM >= L) return;  // this pair of query tiles lies beyond the segment
-  // once any CTA of this launch has given up on a wait, the rest stand down (read only by the
-  // CTAs that have work: the grid is sized by the longest segment, and most of a short
-  // segment's CTAs leave above after their two cu_seqlens loads)
-  if (*reinterpret_cast<volatile int32_t*>(status) == VCS_ERR_DEVICE_TIMEOUT) return;
-  // prefix reuse: the pair's rows equal the previous segment's (copied by fwd_reuse_copy)
-  if (seg_shared != nullptr && (p + 1) * 2 * C::BM <= reuse_skip_rows(seg_shared, cu_seqlens, seg, status)) return;
   const int m0 = 2 * p, m1 = 2 * p + 1;
   const bool has1 = m1 * C::BM < L;
   const int nkv = has1 ? m1 + 1 : m0 + 1;
@@ -512,8 +589,15 @@ __global__ void __launch_bounds__(256) fwd_reuse_copy(const int32_t* __restrict_
   }
 }
 
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Upper bound of a launch's work units: hq * sum_s ceil(L_s / 256) <= hq * (T / 256 + S + 1).
+inline int64_t fwd_max_items(const AttnArgs& a) {
+  return (int64_t)a.hq * (a.num_tokens / 256 + (int64_t)a.num_segments + 1);
+}
+
 template <int D, bool GATHER>
-cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st) {
+cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st) {
   using C = Fwd<D>;
   alignas(64) CUtensorMap tq, tk, tv, tqr, tkr, tvr, tqs, tks, tvs;
   if (GATHER) {
@@ -541,17 +625,22 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
   if (!regs_ok) return cudaErrorInvalidConfiguration;
   cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, GATHER>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (e != cudaSuccess) return e;
-  const int npairs = (a.max_seqlen + 2 * C::BM - 1) / (2 * C::BM);
-  if (npairs == 0) return cudaSuccess;
-  const int64_t gx = (int64_t)a.num_segments * a.hq * npairs;
-  if (gx > INT32_MAX) return cudaErrorInvalidConfiguration;
+  const int64_t max_items = fwd_max_items(a);
+  if (max_items > INT32_MAX) return cudaErrorInvalidConfiguration;
+  // workspace: header (status word, unit count), off[S+1], the units
+  char* w = static_cast<char*>(ws);
+  int32_t* total = reinterpret_cast<int32_t*>(w + kWsItemTotal);
+  int32_t* off = reinterpret_cast<int32_t*>(w + kWsHeader);
+  int4* items = reinterpret_cast<int4*>(w + kWsHeader + align256(((size_t)a.num_segments + 1) * 4));
+  fwd_item_scan<<<1, 1024, 0, st>>>(a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq,
+                                    a.seg_shared, off, total, a.status);
+  const int fill_blocks = a.num_segments < 152 * 8 ? a.num_segments : 152 * 8;
+  fwd_item_fill<<<fill_blocks, 256, 0, st>>>(a.cu_seqlens, a.num_segments, a.hq, a.hkv, off, items);
   const float scale_log2 = a.scale * 1.4426950408889634f;
-  dim3 grid((unsigned)gx, 1, 1);
-  attn_fwd_kernel<D, GATHER><<<grid, kThreads, C::SMEM, st>>>(
-      tq, tk, tv, a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq, a.hkv, npairs, scale_log2,
-      static_cast<__nv_bfloat16*>(o), lse, a.status, a.tok_gather, (int32_t)a.traj_tokens, GATHER ? tqr : tq,
-      GATHER ? tkr : tk, GATHER ? tvr : tv, a.seg_shared, GATHER ? tqs : tq, GATHER ? tks : tk,
-      GATHER ? tvs : tv);
+  attn_fwd_kernel<D, GATHER><<<(unsigned)max_items, kThreads, C::SMEM, st>>>(
+      tq, tk, tv, items, total, (int32_t)a.num_tokens, a.hq, a.hkv, scale_log2, static_cast<__nv_bfloat16*>(o),
+      lse, a.status, a.tok_gather, (int32_t)a.traj_tokens, GATHER ? tqr : tq, GATHER ? tkr : tk,
+      GATHER ? tvr : tv, GATHER ? tqs : tq, GATHER ? tks : tk, GATHER ? tvs : tv);
   if (a.seg_shared != nullptr) {
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -566,19 +655,21 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, cudaStream_t st
 
 }  // namespace
 
+// Header (status word, unit count), the per-segment unit offsets and the list of work units
+// (16 bytes each).
 size_t attn_fwd_ws_bytes(const AttnArgs& a) {
-  (void)a;
-  return kWsHeader;
+  const int64_t items = fwd_max_items(a);
+  return kWsHeader + align256(((size_t)(a.num_segments > 0 ? a.num_segments : 0) + 1) * 4) +
+         align256((size_t)(items > 0 ? items : 0) * 16);
 }
 
 cudaError_t launch_attn_fwd(const AttnArgs& a, void* o, float* lse, void* ws, cudaStream_t st) {
-  (void)ws;
   if (a.tok_gather != nullptr) {
-    if (a.d == 64) return launch_fwd_d<64, true>(a, o, lse, st);
-    return launch_fwd_d<128, true>(a, o, lse, st);
+    if (a.d == 64) return launch_fwd_d<64, true>(a, o, lse, ws, st);
+    return launch_fwd_d<128, true>(a, o, lse, ws, st);
   }
-  if (a.d == 64) return launch_fwd_d<64, false>(a, o, lse, st);
-  return launch_fwd_d<128, false>(a, o, lse, st);
+  if (a.d == 64) return launch_fwd_d<64, false>(a, o, lse, ws, st);
+  return launch_fwd_d<128, false>(a, o, lse, ws, st);
 }
 
 }  // namespace vcs
