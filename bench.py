@@ -277,7 +277,7 @@ class Path:
                 evs[3].record(tstream)
             st = vcs.vcs_attn_fwd(self.q, self.k, self.v, self.cu_seqlens, nseg, ntok, ci["max_seqlen"], hq, hkv,
                                   d, 0.0, self.o, self.lse, self.fwd_ws, self.fwd_ws_bytes, stream)
-            launches += 1
+            launches += 3  # the work-unit scan and fill, then the attention kernel
             assert st == 0
             if evs:
                 evs[4].record(tstream)

@@ -146,3 +146,59 @@ def test_inconsistent_cu_seqlens_reported():
     with pytest.raises(vcs.VcsError) as e:
         vcs.attn_fwd(q, k, v, bad, 64)
     assert e.value.status == 6
+
+
+def _units_of(cu, hq):
+    """Work units the forward lists: hq per 256-row pair of query tiles of each segment."""
+    lens = np.diff(np.asarray(cu, np.int64))
+    return int(hq * ((lens + 255) // 256).sum())
+
+
+def test_work_unit_list_with_empty_segments():
+    # empty segments at the start, in the middle and at the end, and segments that end a
+    # pair of query tiles early or exactly: the listed unit count (workspace header, int32 at
+    # byte 128) is exact, and every row matches the oracle
+    from paper_2607_11185_gb300 import vcs
+    lengths = [0, 0, 300, 0, 256, 1, 0, 513, 257, 0]
+    hq, hkv, d = 5, 1, 128
+    cu = cu_from_lengths(lengths)
+    nt = int(cu[-1])
+    q, k, v, _ = workloads.draw_dense(71, nt, hq, hkv, d, device="cuda")
+    dcu = torch.from_numpy(np.asarray(cu, np.int32)).cuda()
+    ns = len(lengths)
+    nb = vcs.vcs_attn_fwd_workspace_size(ns, nt, max(lengths), hq, hkv, d)
+    assert nb >= 256 + 4 * (ns + 1) + 16 * _units_of(cu, hq)
+    ws = torch.zeros(nb, dtype=torch.uint8, device="cuda")
+    o = torch.empty_like(q)
+    lse = torch.empty((hq, nt), dtype=torch.float32, device="cuda")
+    assert vcs.vcs_attn_fwd(q, k, v, dcu, ns, nt, max(lengths), hq, hkv, d, 0.0, o, lse, ws, nb) == 0
+    torch.cuda.synchronize()
+    hdr = ws[:256].view(torch.int32).cpu().numpy()
+    assert hdr[0] == 0
+    assert hdr[128 // 4] == _units_of(cu, hq)
+    compare_full(q, k, v, cu, o, lse)
+
+
+@pytest.mark.parametrize("window", [1, 3])
+def test_work_unit_count_on_builder_layouts(window):
+    # the 8-trajectory draw laid out step-wise (W = 1: many short segments, the case the list
+    # is for) and with W = 3: the listed unit count is the closed form over the oracle's
+    # segment lengths, and sampled rows match the oracle
+    from paper_2607_11185_gb300 import vcs
+    w = workloads.WORKLOADS["traj8_w3"]
+    cu_s, img, txt = workloads.draw_steps(w)
+    lay = oseg.build(cu_s, img, txt, window, 0)
+    cu = np.asarray(lay["cu_seqlens"], np.int64)
+    nt, ns = int(cu[-1]), len(cu) - 1
+    mx = int(np.diff(cu).max())
+    q, k, v, _ = workloads.draw_dense(5 + window, nt, w.hq, w.hkv, w.d, device="cuda")
+    dcu = torch.from_numpy(cu.astype(np.int32)).cuda()
+    nb = vcs.vcs_attn_fwd_workspace_size(ns, nt, mx, w.hq, w.hkv, w.d)
+    ws = torch.zeros(nb, dtype=torch.uint8, device="cuda")
+    o = torch.empty_like(q)
+    lse = torch.empty((w.hq, nt), dtype=torch.float32, device="cuda")
+    assert vcs.vcs_attn_fwd(q, k, v, dcu, ns, nt, mx, w.hq, w.hkv, w.d, 0.0, o, lse, ws, nb) == 0
+    torch.cuda.synchronize()
+    hdr = ws[:256].view(torch.int32).cpu().numpy()
+    assert hdr[0] == 0 and hdr[128 // 4] == _units_of(cu, w.hq)
+    check_sampled(q, k, v, cu, o, lse, np.random.default_rng(40 + window), n_seg=4, heads=[0, w.hq - 1])
