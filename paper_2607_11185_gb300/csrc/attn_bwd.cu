@@ -517,10 +517,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 //   WG0   warp 0: TMA producer (K and V once, Q/dO 128-row tiles through a 2-stage ring)
 //         warp 1: TMEM allocation and the single MMA-issuing thread
 //   WG1/2 compute in four phases of 32 query columns, warpgroup k taking 16
-//         columns of each: S^T, dP^T -> P^T (bf16, written back to TMEM over the
-//         warpgroup's own dP^T columns: the A operand of dV += P^T dO) and dS^T
-//         (bf16, shared memory: dK += dS^T Q and dQ = dS K); dV and dK over a
-//         phase's columns run while the next phase is computed
+//         columns of each: S^T, dP^T -> P^T and dS^T (bf16, written back to TMEM
+//         over the warpgroup's own 16 dP^T columns, 8 each: the A operands of
+//         dV += P^T dO and dK += dS^T Q, which then read only their B operand
+//         from shared memory) and dS^T once more in shared memory (for
+//         dQ = dS K); dV and dK over a phase's columns run while the next phase
+//         is computed
 //   WG3   dQ drain: once a tile's MMAs are complete, dQ (query rows on TMEM
 //         lanes) is read two 32-column parts at a time and copied into the tile's
 //         freed Q/dO stage, the columns are handed back, and TMA bulk reduce-adds
@@ -530,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // With a 64-query sub-tile and two streams (compute of one stream overlapping
 // the other's MMAs) the N = 64 MMAs held the backward 5% lower on the
 // long-horizon workload than this single stream of 128-query tiles.
-//   TMEM: dV [0,128), dK [128,256); S^T then dQ, and dP^T then P^T, in [256,384) and
+//   TMEM: dV [0,128), dK [128,256); S^T then dQ, and dP^T then P^T/dS^T, in [256,384) and
 //         [384,512), swapping roles every tile so that S^T(u+1) can be computed while
 //         dQ(u) is drained
 //   smem: K, V (64 KB), 2-stage Q/dO ring (128 KB; a freed stage also stages dQ),
@@ -574,7 +576,8 @@ __device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)
 // off-diagonal tiles run a branch-free body the compiler can interleave.
 template <int NC, bool DIAG>
 __device__ __forceinline__ void d128_phase_math(const uint32_t (&sv)[NC], const uint32_t (&pv)[NC],
-                                                uint32_t (&pt)[NC / 2], const uint4 (&rq)[NC / 2], uint64_t sl2,
+                                                uint32_t (&pt)[NC / 2], uint32_t (&dt)[NC / 2],
+                                                const uint4 (&rq)[NC / 2], uint64_t sl2,
                                                 uint64_t sc2, int dlim, uint32_t ds_row, int ch0, int r) {
 #pragma unroll
   for (int ch = 0; ch < NC / 8; ++ch) {
@@ -597,6 +600,7 @@ __device__ __forceinline__ void d128_phase_math(const uint32_t (&sv)[NC], const 
       f2unpack(fmul2(pp, t), d0, d1);
       pt[ch * 4 + e] = pack_bf16(p0, p1);
       wd[e] = pack_bf16(d0, d1);
+      dt[ch * 4 + e] = wd[e];
     }
     st_shared_v4(ds_row + (uint32_t)(((ch0 + ch) ^ (r & 7)) << 4), wd[0], wd[1], wd[2], wd[3]);
   }
@@ -633,6 +637,8 @@ struct D128 {
   __host__ __device__ static constexpr uint32_t pt_col(int kk) {
     return PW * (kk / KPP) + HW * ((kk % KPP) / (KPP / 2)) + 8 * (kk % (KPP / 2));
   }
+  // ... and its dS^T (the A operand of dK += dS^T Q) in the 8 columns after them: each
+  // warpgroup's 16 dP^T columns of a phase hold exactly one K = 16 step of each
   static constexpr int REG_CTRL = 96, REG_COMPUTE = 168, REG_DRAIN = 80;
   static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
@@ -640,6 +646,7 @@ struct D128 {
   static constexpr uint32_t IDESC_DQ = idesc_bf16(128, 128, 1, 1);  // dS (MN-major) x K (MN-major)
 };
 static_assert(D128::SMEM <= 232448, "shared memory budget");
+static_assert(D128::HW == 16, "a warpgroup's phase columns hold one K step of P^T and one of dS^T");
 static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D128::REG_LAUNCH,
               "setmaxnreg targets exceed the registers the block is launched with");
 
@@ -834,7 +841,6 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const uint64_t k_mnmaj = smem_desc(sbase + C::OFF_K, C::BLOCK, 1024);
       const uint64_t q_kmaj = smem_desc(sbase + C::OFF_Q, 16, 1024);
       const uint64_t q_mnmaj = smem_desc(sbase + C::OFF_Q, C::BLOCK, 1024);
-      const uint64_t ds_kmaj = smem_desc(sbase + C::OFF_DS, 16, 1024);
       const uint64_t ds_mnmaj = smem_desc(sbase + C::OFF_DS, C::BLOCK, 1024);
       for (int u = 0; ok && u < U; ++u) {
         const int stage = u % C::NST;
@@ -878,8 +884,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
                       kk > 0 ? 1u : acc0);
 #pragma unroll
           for (int kk = kk0; kk < kk0 + C::KPP; ++kk)
-            tc_mma_ss(tmem + C::TM_DK, desc_at(ds_kmaj, (kk >> 2) * C::BLOCK + (kk & 3) * 32),
-                      desc_at(qmn, kk * 2048), C::IDESC_KV, kk > 0 ? 1u : acc0);
+            tc_mma_ts(tmem + C::TM_DK, cp + C::pt_col(kk) + 8, desc_at(qmn, kk * 2048), C::IDESC_KV,
+                      kk > 0 ? 1u : acc0);
         };
 #pragma unroll
         for (int ph = 0; ph < C::NPH - 1; ++ph) {
@@ -950,9 +956,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
       const bool got = mbar_wait_warp(&bars->s_full, u & 1);
       if (got) {
         tc_fence_after();
-        // phase ph: query columns [PW*ph + HW*k, PW*ph + HW*k + HW); its P^T (HW/2 words) goes
-        // over the first of its own dP^T columns, its dS^T into HW/8 16-byte chunks of the
-        // shared block of its 64 queries
+        // phase ph: query columns [PW*ph + HW*k, PW*ph + HW*k + HW); its P^T and dS^T (HW/2
+        // words each) go over its own dP^T columns, and its dS^T also into HW/8 16-byte chunks
+        // of the shared block of its 64 queries
         // the next phase's S^T and dP^T columns are loaded while this phase is computed
         uint32_t sv[2][C::HW], pv[2][C::HW];
         tmem_ld_cols<C::HW>(trow + C::col_s(u) + C::HW * k, sv[0]);
@@ -972,16 +978,17 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           uint4 rq[C::HW / 2];
 #pragma unroll
           for (int e = 0; e < C::HW / 2; ++e) rq[e] = ld_shared_v4(rt_u32 + (uint32_t)(C::PW * ph + 4 * e) * 4);
-          uint32_t pt[C::HW / 2];
+          uint32_t pt[C::HW / 2], dt[C::HW / 2];
           const uint32_t ds_row = sbase + C::OFF_DS + (col / 64) * C::BLOCK + r * 128;
           const int ch0 = (int)(col % 64) / 8;
           if (diag)
-            d128_phase_math<C::HW, true>(sv[cur], pv[cur], pt, rq, sl2, sc2, r - (int)col, ds_row, ch0, r);
+            d128_phase_math<C::HW, true>(sv[cur], pv[cur], pt, dt, rq, sl2, sc2, r - (int)col, ds_row, ch0, r);
           else
-            d128_phase_math<C::HW, false>(sv[cur], pv[cur], pt, rq, sl2, sc2, 0, ds_row, ch0, r);
+            d128_phase_math<C::HW, false>(sv[cur], pv[cur], pt, dt, rq, sl2, sc2, 0, ds_row, ch0, r);
           // dS^T (shared memory) is published to the tensor pipe while P^T's TMEM store completes
           fence_proxy_async_smem();
           tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col, pt);
+          tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col + C::HW / 2, dt);
           tmem_st_wait();
           tc_fence_before();
           mbar_arrive(&bars->p_full[ph]);
