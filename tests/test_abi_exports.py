@@ -109,3 +109,20 @@ def test_selftest_bounded_wait_argument_errors_without_gpu(lib):
     assert f(256, 0, None) == 1
     assert f(256, -5, None) == 1
     assert f(256, 4_000_000_001, None) == 1
+
+
+def test_forward_workspace_holds_the_unit_list(lib):
+    # header, per-segment unit offsets, then 16 bytes per work unit: at most
+    # hq * (num_tokens / 256 + num_segments + 1) units, which bounds hq * sum_s ceil(L_s / 256)
+    import numpy as np
+    f = lib.vcs_attn_fwd_workspace_size
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_int32, ctypes.c_int64] + [ctypes.c_int32] * 4
+    r256 = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    for s, t, hq in ((1, 10, 2), (56, 1_972_928, 40), (1040, 7_727_164, 40), (5, 0, 8)):
+        assert f(s, t, 4096, hq, 1, 128) == 256 + r256((s + 1) * 4) + r256(hq * (t // 256 + s + 1) * 16)
+    rng = np.random.default_rng(0)
+    for _ in range(500):
+        lens = rng.integers(0, 5000, size=int(rng.integers(1, 60)))
+        t, s = int(lens.sum()), len(lens)
+        assert int(((lens + 255) // 256).sum()) <= t // 256 + s + 1
