@@ -154,7 +154,9 @@ vcs_status vcs_gather(const void* q_traj, const void* k_traj, const void* v_traj
  * most hq * (num_tokens / 256 + num_segments + 1) of them) and their
  * per-segment offsets, built on the device by the call itself; about
  * hq * num_tokens / 16 bytes.  Also the size for vcs_attn_fwd_reuse and
- * vcs_attn_fwd_gathered. */
+ * vcs_attn_fwd_gathered.  Inconsistent cu_seqlens can describe overlapping
+ * segments with more units than that: then no unit runs (nothing is written
+ * past the list) and the status word reports VCS_ERR_DEVICE_CHECK. */
 size_t vcs_attn_fwd_workspace_size(int32_t num_segments, int64_t num_tokens, int32_t max_seqlen,
                                    int32_t hq, int32_t hkv, int32_t d);
 

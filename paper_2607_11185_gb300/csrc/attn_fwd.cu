@@ -160,65 +160,75 @@ __device__ __forceinline__ int seg_item_pairs(const int32_t* __restrict__ cu_seq
 }
 
 // off[s] = hq * (pairs of segments 0 .. s-1), off[S] = *total: one block, in chunks of 1024
-// segments (warp scans, then a scan of the warp sums).
+// segments (warp scans, then a scan of the warp sums), in 64-bit.  Consistent segments list at
+// most `capacity` units (the workspace's room); segments that overlap, which only inconsistent
+// bounds allow, can list more: the offsets are then clipped to the capacity, the count is 0 (no
+// unit runs, so no CTA reads a unit the fill did not write) and the call records
+// VCS_ERR_DEVICE_CHECK (already recorded for the inconsistent segment).
 __global__ void __launch_bounds__(1024) fwd_item_scan(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
                                                       int32_t num_tokens, int32_t max_seqlen, int32_t hq,
-                                                      const int32_t* __restrict__ seg_shared,
+                                                      const int32_t* __restrict__ seg_shared, int32_t capacity,
                                                       int32_t* __restrict__ off, int32_t* __restrict__ total,
                                                       int32_t* status) {
-  __shared__ int32_t wsum[32];
-  __shared__ int32_t carry;
+  __shared__ long long wsum[32];
+  __shared__ long long carry;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
   for (int base = 0; base < num_segments; base += 1024) {
     const int s = base + (int)threadIdx.x;
-    const int cnt =
-        s < num_segments ? hq * seg_item_pairs(cu_seqlens, num_segments, num_tokens, max_seqlen, seg_shared, s, status)
-                         : 0;
-    int x = cnt;
+    const long long cnt =
+        s < num_segments
+            ? (long long)hq * seg_item_pairs(cu_seqlens, num_segments, num_tokens, max_seqlen, seg_shared, s, status)
+            : 0;
+    long long x = cnt;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      const long long y = __shfl_up_sync(0xffffffffu, x, o);
       if (lane >= o) x += y;
     }
     if (lane == 31) wsum[wid] = x;
     __syncthreads();
     if (wid == 0) {
-      int w = wsum[lane];
+      long long w = wsum[lane];
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, w, o);
+        const long long y = __shfl_up_sync(0xffffffffu, w, o);
         if (lane >= o) w += y;
       }
       wsum[lane] = w;
     }
     __syncthreads();
-    const int incl = carry + (wid > 0 ? wsum[wid - 1] : 0) + x;
-    if (s < num_segments) off[s] = incl - cnt;
+    const long long incl = carry + (wid > 0 ? wsum[wid - 1] : 0) + x;
+    if (s < num_segments) off[s] = (int32_t)(incl - cnt < capacity ? incl - cnt : capacity);
     __syncthreads();
     if (threadIdx.x == 1023) carry = incl;
     __syncthreads();
   }
   if (threadIdx.x == 0) {
-    off[num_segments] = carry;
-    *total = carry;
+    const int32_t t = carry <= capacity ? (int32_t)carry : 0;
+    if (carry > capacity) set_status(status, VCS_ERR_DEVICE_CHECK);
+    off[num_segments] = t;
+    *total = t;
   }
 }
 
 // The units of segment s at off[s] .. off[s+1]-1, in the order (kv head, pair from the last,
-// query head in the group): {segment start, segment end, pair index, query head}.
+// query head in the group): {segment start, segment end, pair index, query head}.  A segment
+// whose units would not all fit in the capacity (clipped by fwd_item_scan) writes none.
 __global__ void __launch_bounds__(256) fwd_item_fill(const int32_t* __restrict__ cu_seqlens, int32_t num_segments,
-                                                     int32_t hq, int32_t hkv, const int32_t* __restrict__ off,
-                                                     int4* __restrict__ items) {
+                                                     int32_t num_tokens, int32_t max_seqlen, int32_t hq, int32_t hkv,
+                                                     const int32_t* __restrict__ seg_shared, int32_t capacity,
+                                                     const int32_t* __restrict__ off, int4* __restrict__ items,
+                                                     int32_t* status) {
   const int G = hq / hkv;
   for (int s = blockIdx.x; s < num_segments; s += gridDim.x) {
-    const int base = off[s], n = off[s + 1] - base;
-    if (n == 0) continue;
+    const int cnt = seg_item_pairs(cu_seqlens, num_segments, num_tokens, max_seqlen, seg_shared, s, status);
+    const long long base = off[s], n = (long long)hq * cnt;
+    if (cnt == 0 || base + n > capacity) continue;
     const int start = cu_seqlens[s], end = cu_seqlens[s + 1];
-    const int np = (end - start + 255) / 256;
-    const int cnt = n / hq;  // pairs np - cnt .. np - 1
-    for (int r = threadIdx.x; r < n; r += blockDim.x) {
+    const int np = (end - start + 255) / 256;  // pairs np - cnt .. np - 1
+    for (int r = threadIdx.x; r < (int)n; r += blockDim.x) {
       const int hh = r % G, r2 = r / G;
       const int pr = r2 % cnt, g = r2 / cnt;
       items[base + r] = make_int4(start, end, np - 1 - pr, g * G + hh);
@@ -226,11 +236,6 @@ __global__ void __launch_bounds__(256) fwd_item_fill(const int32_t* __restrict__
   }
 }
 
-// GATHER: Q, K and V are trajectory-layout tensors read through tok_gather, one warp per
-// tile: tm_q/k/v are 2-D maps of 64 x 1 boxes for TMA gather4 loads, tm_qr/kr/vr and
-// tm_qs/ks/vs 3-D tiled maps of the same tensors (128- and 32-row boxes) for tiles or
-// 32-row groups whose rows are consecutive trajectory rows.  Otherwise tm_q/k/v are
-// segment-layout tiled maps and the others are unused.
 template <int D, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -633,9 +638,10 @@ cudaError_t launch_fwd_d(const AttnArgs& a, void* o, float* lse, void* ws, cudaS
   int32_t* off = reinterpret_cast<int32_t*>(w + kWsHeader);
   int4* items = reinterpret_cast<int4*>(w + kWsHeader + align256(((size_t)a.num_segments + 1) * 4));
   fwd_item_scan<<<1, 1024, 0, st>>>(a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen, a.hq,
-                                    a.seg_shared, off, total, a.status);
+                                    a.seg_shared, (int32_t)max_items, off, total, a.status);
   const int fill_blocks = a.num_segments < 152 * 8 ? a.num_segments : 152 * 8;
-  fwd_item_fill<<<fill_blocks, 256, 0, st>>>(a.cu_seqlens, a.num_segments, a.hq, a.hkv, off, items);
+  fwd_item_fill<<<fill_blocks, 256, 0, st>>>(a.cu_seqlens, a.num_segments, (int32_t)a.num_tokens, a.max_seqlen,
+                                             a.hq, a.hkv, a.seg_shared, (int32_t)max_items, off, items, a.status);
   const float scale_log2 = a.scale * 1.4426950408889634f;
   attn_fwd_kernel<D, GATHER><<<(unsigned)max_items, kThreads, C::SMEM, st>>>(
       tq, tk, tv, items, total, (int32_t)a.num_tokens, a.hq, a.hkv, scale_log2, static_cast<__nv_bfloat16*>(o),

@@ -148,6 +148,32 @@ def test_inconsistent_cu_seqlens_reported():
     assert e.value.status == 6
 
 
+@pytest.mark.parametrize("bounds,expect_units", [
+    # overlapping segments that fit the unit list: both run (over the same rows), the bad one
+    # in between is reported
+    ([0, 512, 0, 512], 2 * (2 + 2)),
+    # five full-length segments over the same 16,384 rows: 640 units against room for 148, so
+    # none runs (nothing is written past the list) and the call reports the check
+    ([0, 16384, 0, 16384, 0, 16384, 0, 16384, 0, 16384], 0),
+])
+def test_overlapping_segments_reported_and_bounded(bounds, expect_units):
+    from paper_2607_11185_gb300 import vcs
+    nt = bounds[-1]
+    hq, hkv, d = 2, 1, 64
+    q, k, v, _ = workloads.draw_dense(2, nt, hq, hkv, d, device="cuda")
+    cu = torch.tensor(bounds, dtype=torch.int32, device="cuda")
+    ns = len(bounds) - 1
+    nb = vcs.vcs_attn_fwd_workspace_size(ns, nt, nt, hq, hkv, d)
+    ws = torch.zeros(nb, dtype=torch.uint8, device="cuda")
+    o = torch.zeros_like(q)
+    lse = torch.zeros((hq, nt), dtype=torch.float32, device="cuda")
+    assert vcs.vcs_attn_fwd(q, k, v, cu, ns, nt, nt, hq, hkv, d, 0.0, o, lse, ws, nb) == 0
+    torch.cuda.synchronize()
+    hdr = ws[:256].view(torch.int32).cpu().numpy()
+    assert hdr[0] == 6
+    assert hdr[128 // 4] == expect_units
+
+
 def _units_of(cu, hq):
     """Work units the forward lists: hq per 256-row pair of query tiles of each segment."""
     lens = np.diff(np.asarray(cu, np.int64))
