@@ -569,9 +569,9 @@ __device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)
 //   P^T  = 2^(S^T * scale*log2e - lse*log2e)     (zero where the key follows the query)
 //   dS^T = P^T * (dP^T - D) * scale
 // The row terms come as {-lse*log2e, -D*scale} of each column pair, one 16-byte load
-// {nl(c), nl(c+1), nd(c), nd(c+1)} per pair.  P^T goes to pt as bf16 pairs; dS^T to
-// 16-byte chunks CH0 .. CH0+NC/8-1 of the thread's 128-byte row of the swizzled K-major
-// shared block.  The causal test is compiled
+// {nl(c), nl(c+1), nd(c), nd(c+1)} per pair.  P^T goes to pt and dS^T to dt as bf16 pairs
+// (for TMEM), and dS^T also to 16-byte chunks CH0 .. CH0+NC/8-1 of the thread's 128-byte row
+// of the swizzled K-major shared block.  The causal test is compiled
 // only into the diagonal instantiation (column c is masked when c < dlim), so the
 // off-diagonal tiles run a branch-free body the compiler can interleave.
 template <int NC, bool DIAG>
@@ -642,7 +642,7 @@ struct D128 {
   static constexpr int REG_CTRL = 96, REG_COMPUTE = 168, REG_DRAIN = 80;
   static constexpr int REG_LAUNCH = 65536 / THREADS;
   static constexpr uint32_t IDESC_S = idesc_bf16(128, 128, 0, 0);   // K or V (K-major) x Q or dO (K-major)
-  static constexpr uint32_t IDESC_KV = idesc_bf16(128, 128, 0, 1);  // P^T (TMEM) / dS^T (K-major) x dO / Q (MN-major)
+  static constexpr uint32_t IDESC_KV = idesc_bf16(128, 128, 0, 1);  // P^T / dS^T (TMEM) x dO / Q (MN-major)
   static constexpr uint32_t IDESC_DQ = idesc_bf16(128, 128, 1, 1);  // dS (MN-major) x K (MN-major)
 };
 static_assert(D128::SMEM <= 232448, "shared memory budget");
@@ -874,7 +874,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
         // dV += P^T dO and dK += dS^T Q over each phase's queries as soon as they are written
         // (overlapping the compute of the next phase), then, after the last phase, dQ = dS K
         // and the last phase's dV, dK.  In-order execution keeps S(u+1) from overwriting P^T or
-        // dS^T first.  P^T of queries [16kk, 16kk+16) sits at C::pt_col(kk) of its columns.
+        // dS^T first.  P^T of queries [16kk, 16kk+16) sits at C::pt_col(kk) of its columns, their
+        // dS^T 8 columns further.
         const uint64_t qmn = desc_at(q_mnmaj, stage * 2 * C::TILE), dmn = desc_at(qmn, C::TILE);
         const uint32_t acc0 = u > 0 ? 1u : 0u;
         auto issue_dvdk = [&](int kk0) {
@@ -985,7 +986,8 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
             d128_phase_math<C::HW, true>(sv[cur], pv[cur], pt, dt, rq, sl2, sc2, r - (int)col, ds_row, ch0, r);
           else
             d128_phase_math<C::HW, false>(sv[cur], pv[cur], pt, dt, rq, sl2, sc2, 0, ds_row, ch0, r);
-          // dS^T (shared memory) is published to the tensor pipe while P^T's TMEM store completes
+          // dS^T (shared memory) is published to the tensor pipe while the TMEM stores of P^T and
+          // dS^T complete
           fence_proxy_async_smem();
           tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col, pt);
           tmem_st_cols<C::HW / 2>(trow + C::col_p(u) + col + C::HW / 2, dt);
