@@ -40,7 +40,10 @@
 // executes in order, so the completion of S_k(j+1) also means that P_k(j) has
 // been consumed and O_k is up to date, which is all the softmax warps wait
 // for.  The two tiles alternate, so one tile's MMAs run while the other
-// tile's softmax warps work.
+// tile's softmax warps work.  The MMA thread commits only what the softmax
+// warps wait for (a commit holds it, and the pipe, about as long as an MMA);
+// the K/V ring slots are handed back to the producer by one softmax thread of
+// the last tile, whose S(j+1) completing means their reads are done.
 //
 // Online softmax with a lazy running maximum: the row maximum used for P is
 // only raised (and O, l rescaled) when a new tile's maximum exceeds it by more
@@ -387,7 +390,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_s<D>(tmem + C::TM_S1, q1d, desc_at(kv_kmaj, kaddr));
           tc_commit(&bars->s_full[1]);
         }
-        tc_commit(&bars->kv_empty[0]);
       }
       // V_0 and K_1 for the first step; every later step's V and K are acquired one step
       // ahead, between the two tiles' issues, while the tensor pipe still has queued work
@@ -423,8 +425,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_commit(&bars->o_done[1]);
           }
         }
-        if (next) tc_commit(&bars->kv_empty[k_item(j + 1) % C::NSLOT]);
-        tc_commit(&bars->kv_empty[v_item(j) % C::NSLOT]);
         vaddr = vaddr_next;
         kaddr = kaddr_next;
       }
@@ -444,10 +444,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t sc2 = f2pack(scale_log2, scale_log2);
       float m_run = -FLT_MAX, l = 0.f;
       bool ok = true;
+      // The K/V ring slots are handed back from here rather than by commits of the MMA thread
+      // (a tcgen05.commit holds that thread, and the tensor pipe, for about as long as an MMA):
+      // once S_k(j) of the last tile is complete, in-order execution has also completed every
+      // MMA that reads K_j (the S(j) of both tiles) and V_{j-1} (the P V of both tiles at
+      // step j-1), so one thread of that tile's warpgroup frees their slots.  The last V_{n-1}
+      // is not handed back: the producer has issued every load by then.
+      const bool releaser = (has1 ? wg == 1 : wg == 0) && quad == 0 && lane == 0;
       for (int j = 0; j <= mt; ++j) {
         // S(j) complete also means P(j-1) was consumed and O holds P(j-1) V.  The wait's
         // outcome is the warp's: the TMEM loads and votes below are warp-collective.
         if (!mbar_wait_warp(&bars->s_full[wg], j & 1)) { ok = false; break; }
+        if (releaser) {
+          mbar_arrive(&bars->kv_empty[(j == 0 ? 0 : 2 * j - 1) % C::NSLOT]);                  // K_j
+          if (j > 0) mbar_arrive(&bars->kv_empty[(j - 1 == nkv - 1 ? 2 * nkv - 1 : 2 * j) % C::NSLOT]);  // V_{j-1}
+        }
         tc_fence_after();
         uint32_t s[128];
 #pragma unroll
