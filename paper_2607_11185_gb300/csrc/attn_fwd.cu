@@ -43,7 +43,9 @@
 // tile's softmax warps work.  The MMA thread commits only what the softmax
 // warps wait for (a commit holds it, and the pipe, about as long as an MMA);
 // the K/V ring slots are handed back to the producer by one softmax thread of
-// the last tile, whose S(j+1) completing means their reads are done.
+// the last tile, whose S(j+1) completing means their reads are done.  (The
+// gathered variant, whose producer issues its loads more slowly, has them
+// handed back by commits as soon as the MMAs are done.)
 //
 // Online softmax with a lazy running maximum: the row maximum used for P is
 // only raised (and O, l rescaled) when a new tile's maximum exceeds it by more
@@ -390,6 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_s<D>(tmem + C::TM_S1, q1d, desc_at(kv_kmaj, kaddr));
           tc_commit(&bars->s_full[1]);
         }
+        if constexpr (GATHER) tc_commit(&bars->kv_empty[0]);
       }
       // V_0 and K_1 for the first step; every later step's V and K are acquired one step
       // ahead, between the two tiles' issues, while the tensor pipe still has queued work
@@ -425,6 +428,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_commit(&bars->o_done[1]);
           }
         }
+        if constexpr (GATHER) {
+          // the gathering producer needs its slots back as soon as the MMAs are done with them
+          if (next) tc_commit(&bars->kv_empty[k_item(j + 1) % C::NSLOT]);
+          tc_commit(&bars->kv_empty[v_item(j) % C::NSLOT]);
+        }
         vaddr = vaddr_next;
         kaddr = kaddr_next;
       }
@@ -450,7 +458,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // MMA that reads K_j (the S(j) of both tiles) and V_{j-1} (the P V of both tiles at
       // step j-1), so one thread of that tile's warpgroup frees their slots.  The last V_{n-1}
       // is not handed back: the producer has issued every load by then.
-      const bool releaser = (has1 ? wg == 1 : wg == 0) && quad == 0 && lane == 0;
+      const bool releaser = !GATHER && (has1 ? wg == 1 : wg == 0) && quad == 0 && lane == 0;
       for (int j = 0; j <= mt; ++j) {
         // S(j) complete also means P(j-1) was consumed and O holds P(j-1) V.  The wait's
         // outcome is the warp's: the TMEM loads and votes below are warp-collective.
