@@ -464,8 +464,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // outcome is the warp's: the TMEM loads and votes below are warp-collective.
         if (!mbar_wait_warp(&bars->s_full[wg], j & 1)) { ok = false; break; }
         if (releaser) {
-          mbar_arrive(&bars->kv_empty[(j == 0 ? 0 : 2 * j - 1) % C::NSLOT]);                  // K_j
-          if (j > 0) mbar_arrive(&bars->kv_empty[(j - 1 == nkv - 1 ? 2 * nkv - 1 : 2 * j) % C::NSLOT]);  // V_{j-1}
+          // ring items: K_j is 0 for j = 0, else 2j-1; V_{j-1} is 2(j-1)+2 = 2j (j-1 < nkv-1 here)
+          mbar_arrive(&bars->kv_empty[(j == 0 ? 0 : 2 * j - 1) % C::NSLOT]);
+          if (j > 0) mbar_arrive(&bars->kv_empty[(2 * j) % C::NSLOT]);
         }
         tc_fence_after();
         uint32_t s[128];
