@@ -579,7 +579,8 @@ def main():
         "attn_fwd_ms": fwd_ms, "attn_bwd_ms": bwd_ms,
         "attn_fwd_tflops": f_fwd / (fwd_ms / 1e3) / 1e12, "attn_bwd_tflops": f_bwd / (bwd_ms / 1e3) / 1e12,
         "attn_fwdbwd_tflops": flops / ((fwd_ms + bwd_ms) / 1e3) / 1e12,
-        "frac_of_bf16_burst": value / burst, "frac_of_bf16_sustained": value / sustained,
+        # the job's rate against the job's peak: N GPUs' worth
+        "frac_of_bf16_burst": value / (world * burst), "frac_of_bf16_sustained": value / (world * sustained),
         "flash_convention_tflops": value * 14.0 / 12.0,
         "segment_tokens_per_s": job_tokens / (ms / 1e3),
         "roofline": {"bound": "tensor", "kernel": "vcs_attn_bwd (bwd_pre + bwd_main + bwd_dq_cvt)",
@@ -595,7 +596,7 @@ def main():
         "fused_gather": fused,
         "prefix_reuse": reuse,
         "hbm_kernels": hbm_kernels,
-        "gpu_launches": path.launches_per_step * args.steps,
+        "gpu_launches": int(sum_over_ranks(float(path.launches_per_step * args.steps), dev)),  # every rank's
         "clocks": ck,
     }
     if rank == 0:
@@ -978,6 +979,9 @@ def run_e2e(path, args, flops, stream):
     r0 = ci["tok0"] if whole else 0
     for name, dev_t in zip(("dq", "dk", "dv"), gsets[state["last"][1]]):
         assert torch.equal(res[name][r0 + n - 1], dev_t[n - 1].cpu()), name
+    # the bytes every rank copies (the whole job's, like the value)
+    h2d = sum_over_ranks(float(h2d), path.dev)
+    d2h = sum_over_ranks(float(d2h), path.dev)
     return {"value": flops / (ms / 1e3) / 1e12, "unit": "TFLOP/s", "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "result": "dQ, dK, dV of every segment token (bf16) copied to pinned host memory every step, into "
