@@ -45,7 +45,10 @@
 // the K/V ring slots are handed back to the producer by one softmax thread of
 // the last tile, whose S(j+1) completing means their reads are done.  (The
 // gathered variant, whose producer issues its loads more slowly, has them
-// handed back by commits as soon as the MMAs are done.)
+// handed back by commits as soon as the MMAs are done.)  The ring order puts
+// the two tiles step j reads, K_{j+1} and V_j, next to each other, so the
+// tiled loads complete one barrier per step and the MMA thread waits once a
+// step for its K/V, at the top of the step.
 //
 // Online softmax with a lazy running maximum: the row maximum used for P is
 // only raised (and O, l rescaled) when a new tile's maximum exceeds it by more
@@ -77,6 +80,7 @@ struct Fwd {
   static constexpr int TILE = BM * D * 2;           // bytes of a 128 x D bf16 tile
   static constexpr int BLOCK = BM * 128;            // bytes of one 128 x 64 column block
   static constexpr int NSLOT = 5;
+  static constexpr int NGRP = 4;                    // ring-item group barriers (tiled loads)
   static constexpr int OFF_Q0 = 0;
   static constexpr int OFF_Q1 = TILE;
   static constexpr int OFF_KV = 2 * TILE;
@@ -90,8 +94,9 @@ static_assert(Fwd<128>::SMEM <= 232448, "shared memory budget");
 
 struct Bars {
   uint64_t q_full;
-  uint64_t kv_full[5];
+  uint64_t kv_full[5];   // per ring slot (gathered loads)
   uint64_t kv_empty[5];
+  uint64_t grp_full[4];  // per pair of ring items consumed in one step (tiled loads)
   uint64_t s_full[2];
   uint64_t p_full[2];
   uint64_t o_done[2];
@@ -280,6 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->kv_full[i], 1);
       mbar_init(&bars->kv_empty[i], 1);
     }
+    for (int i = 0; i < C::NGRP; ++i) mbar_init(&bars->grp_full[i], 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->s_full[i], 1);
       mbar_init(&bars->p_full[i], 128);
@@ -357,12 +363,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           if (aborted(bars)) break;
-          mbar_arrive_expect_tx(&bars->kv_full[slot], C::TILE);
+          // items 2m-1, 2m (K_m, V_{m-1}) are the ones step m-1 consumes: they complete one
+          // barrier, armed for both by the first; group 0 (K_0) and group nkv (V_{nkv-1})
+          // hold one item
+          const int m = (c + 1) >> 1;
+          uint64_t* gb = &bars->grp_full[m % C::NGRP];
+          if (c == 0 || (c & 1)) mbar_arrive_expect_tx(gb, (m == 0 || m == nkv ? 1 : 2) * C::TILE);
           const CUtensorMap* tm = is_v ? &tm_v : &tm_k;
 #pragma unroll
           for (int kb = 0; kb < C::KB; ++kb)
-            tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, &bars->kv_full[slot], kb * 64, g,
-                             start + j * C::BN, keep_l2);
+            tma_load_3d_hint(smem + C::OFF_KV + slot * C::TILE + kb * C::BLOCK, tm, gb, kb * 64, g, start + j * C::BN,
+                             keep_l2);
         }
       }
     } else if (warp == 1 && lane == 0) {
@@ -372,19 +383,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t q0d = smem_desc(sbase + C::OFF_Q0, 16, 1024), q1d = desc_at(q0d, C::TILE);
       const uint64_t kv_kmaj = smem_desc(sbase + C::OFF_KV, 16, 1024);
       const uint64_t kv_mnmaj = smem_desc(sbase + C::OFF_KV, C::BLOCK, 1024);
-      // wait for ring item c; returns the byte offset of its slot
-      auto acquire = [&](int c, uint32_t& slot_off) -> bool {
-        const int slot = c % C::NSLOT;
-        if (!mbar_wait(&bars->kv_full[slot], (c / C::NSLOT) & 1)) return false;
-        tc_fence_after();
-        slot_off = slot * C::TILE;
-        return true;
-      };
-      // positions of K_j and V_j in the producer's ring order
+      // positions of K_j and V_j in the producer's ring order, and their slots' byte offsets
       auto k_item = [&](int j) { return j == 0 ? 0 : 2 * j - 1; };
       auto v_item = [&](int j) { return j == nkv - 1 ? 2 * nkv - 1 : 2 * j + 2; };
-      uint32_t kaddr = 0, vaddr = 0;  // slot byte offsets of K_{j+1} and V_j
-      if (ok) ok = acquire(0, kaddr);
+      auto k_off = [&](int j) { return (uint32_t)((k_item(j) % C::NSLOT) * C::TILE); };
+      auto v_off = [&](int j) { return (uint32_t)((v_item(j) % C::NSLOT) * C::TILE); };
+      // tiled loads: group m holds K_m and V_{m-1} (group 0 only K_0, group nkv only
+      // V_{nkv-1}); gathered loads: one barrier per ring item
+      auto acquire_group = [&](int m) -> bool {
+        if constexpr (GATHER) {
+          if (m < nkv && !mbar_wait(&bars->kv_full[k_item(m) % C::NSLOT], (k_item(m) / C::NSLOT) & 1)) return false;
+          if (m > 0 && !mbar_wait(&bars->kv_full[v_item(m - 1) % C::NSLOT], (v_item(m - 1) / C::NSLOT) & 1))
+            return false;
+        } else {
+          if (!mbar_wait(&bars->grp_full[m % C::NGRP], (m / C::NGRP) & 1)) return false;
+        }
+        tc_fence_after();
+        return true;
+      };
+      uint32_t kaddr = k_off(0), vaddr = 0;  // slot byte offsets of K_{j+1} and V_j
+      if (ok) ok = acquire_group(0);
       if (ok) {
         issue_s<D>(tmem + C::TM_S0, q0d, desc_at(kv_kmaj, kaddr));
         tc_commit(&bars->s_full[0]);
@@ -394,14 +412,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if constexpr (GATHER) tc_commit(&bars->kv_empty[0]);
       }
-      // V_0 and K_1 for the first step; every later step's V and K are acquired one step
-      // ahead, between the two tiles' issues, while the tensor pipe still has queued work
-      // (a barrier wait costs hundreds of cycles while the pipe streams from shared memory)
-      uint32_t vaddr_next = 0, kaddr_next = 0;
-      if (ok) ok = acquire(v_item(0), vaddr);
-      if (ok && nkv > 1) ok = acquire(k_item(1), kaddr);
+      // step j reads V_j and K_{j+1}, one group: acquired at the top of the step, one wait a
+      // step (a barrier wait stalls the issuing thread for hundreds of cycles while the pipe
+      // streams from shared memory, so the fewer the better), a step after the producer asked
+      // for it
       for (int j = 0; ok && j < nkv; ++j) {
         const bool next = j + 1 < nkv;
+        if (!acquire_group(j + 1)) { ok = false; break; }
+        vaddr = v_off(j);
+        if (next) kaddr = k_off(j + 1);
         // tile 0: O0 += P0(j) V_j, then S0(j+1)
         if (j <= m0) {
           if (!mbar_wait(&bars->p_full[0], j & 1)) { ok = false; break; }
@@ -414,8 +433,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_commit(&bars->o_done[0]);
           }
         }
-        if (next && !acquire(v_item(j + 1), vaddr_next)) { ok = false; break; }
-        if (j + 2 < nkv && !acquire(k_item(j + 2), kaddr_next)) { ok = false; break; }
         // tile 1
         if (has1) {
           if (!mbar_wait(&bars->p_full[1], j & 1)) { ok = false; break; }
@@ -433,8 +450,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (next) tc_commit(&bars->kv_empty[k_item(j + 1) % C::NSLOT]);
           tc_commit(&bars->kv_empty[v_item(j) % C::NSLOT]);
         }
-        vaddr = vaddr_next;
-        kaddr = kaddr_next;
       }
       if (!ok) on_timeout(bars, status);
     }
