@@ -653,13 +653,13 @@ static_assert(D128::REG_CTRL + 2 * D128::REG_COMPUTE + D128::REG_DRAIN <= 4 * D1
 struct D128Bars {
   uint64_t kv_full;
   uint64_t q_full[D128::NST];      // Q of the stage's tile has landed
-  uint64_t do_full[D128::NST];     // dO of the stage's tile has landed
+  uint64_t do_full[D128::NST];     // dO of the stage's tile has landed and the drain has read the
+                                   // previous tile's dQ out of TMEM (its columns take dP^T next)
   uint64_t kv_done[D128::NST];     // the tile's MMAs are complete: its Q/dO stage may be overwritten
   uint64_t q_free[D128::NST];      // the drain's reduce-adds have read the stage's Q half
   uint64_t do_free[D128::NST];     // ... and its dO half
   uint64_t s_full;
   uint64_t p_full[D128::NPH];  // the query columns of phase ph of the tile: P^T and dS^T written
-  uint64_t tmem_free;
   uint64_t acc_done;
   uint32_t tmem_base;
   int32_t abort;
@@ -720,14 +720,13 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     mbar_init(&bars->kv_full, 1);
     for (int i = 0; i < C::NST; ++i) {
       mbar_init(&bars->q_full[i], 1);
-      mbar_init(&bars->do_full[i], 1);
+      mbar_init(&bars->do_full[i], 1 + 128);  // the producer's bytes + the drain's 128 threads
       mbar_init(&bars->kv_done[i], 1);
       mbar_init(&bars->q_free[i], 1);
       mbar_init(&bars->do_free[i], 1);
     }
     mbar_init(&bars->s_full, 1);
     for (int i = 0; i < C::NPH; ++i) mbar_init(&bars->p_full[i], 256);
-    mbar_init(&bars->tmem_free, 128);
     mbar_init(&bars->acc_done, 1);
     bars->abort = 0;
     fence_mbar_init();
@@ -858,9 +857,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           const uint32_t o = (kk >> 2) * C::BLOCK + (kk & 3) * 32;
           tc_mma_ss(cs, desc_at(k_kmaj, o), desc_at(qd, o), C::IDESC_S, kk > 0);
         }
-        // dP^T = V dO^T goes where dQ(u-1) was: wait for the drain to have read it
-        if ((u > 0 && !mbar_wait(&bars->tmem_free, (u - 1) & 1)) ||
-            !mbar_wait(&bars->do_full[stage], (u / C::NST) & 1)) {
+        // dP^T = V dO^T goes where dQ(u-1) was: one wait for dO and for the drain to have read
+        // dQ(u-1)
+        if (!mbar_wait(&bars->do_full[stage], (u / C::NST) & 1)) {
           ok = false;
           break;
         }
@@ -1059,6 +1058,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
     const int dw = threadIdx.x - 12 * 32;
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
     bool ok = true;
+    // each tile's dP^T waits, with its dO, for the drain to have read the previous tile's dQ;
+    // tile 0 has none
+    mbar_arrive(&bars->do_full[0]);
     for (int u = 0; u < U; ++u) {
       const int stage = u % C::NST;
       const bool got = mbar_wait_warp(&bars->kv_done[stage], (u / C::NST) & 1);
@@ -1076,9 +1078,9 @@ __global__ void __launch_bounds__(D128::THREADS, 1)
           tmem_ld_wait();
           reg_fence<32>(a[0]);
           reg_fence<32>(a[1]);
-          if (pp == D / 64 - 1) {
+          if (pp == D / 64 - 1 && u + 1 < U) {
             tc_fence_before();
-            mbar_arrive(&bars->tmem_free);
+            mbar_arrive(&bars->do_full[(u + 1) % C::NST]);
           }
 #pragma unroll
           for (int i = 0; i < 2; ++i)
